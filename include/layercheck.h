@@ -1,0 +1,291 @@
+/*
+ * layercheck.h -- C ABI of the GB300 LayerCheck hot path (liblayercheck.so).
+ *
+ * LayerCheck (adaptive layer-wise checkpointing, §3) persists at every
+ * checkpoint opportunity only the layers whose normalized weight drift has
+ * reached a threshold, plus any layer that has gone S_max steps without
+ * persistence; each persisted layer carries its weights and their Adam
+ * moments; recovery assembles, per layer, the latest persisted version.
+ *
+ * This library runs the per-step path on one GPU:
+ *   lc_measure   §3.2 Eq. 1   per-layer normalized update u_l (sm_103a kernel)
+ *   lc_select    §3.2 Eq. 2-4 and §3.3 staleness guard (sm_103a kernel)
+ *   lc_pack_*    §3.1 full layer state of the selected layers into one
+ *                contiguous packed stream, optionally on to pinned host memory
+ *   lc_commit_snapshot        reference snapshot <- weights, selected layers
+ *   lc_restore   §3.5 / Eq. 8 mixed-timestamp composite back into place
+ *
+ * Conventions for every call:
+ *   - Every entry point returns lc_status; LC_OK is 0.  On any other value
+ *     lc_last_error() returns a message (thread-local, valid until the next
+ *     call on the same thread).  No call throws or aborts.
+ *   - "device" pointers are CUDA device (or managed) memory of the context's
+ *     device; "host" pointers are ordinary host memory unless stated.
+ *   - The caller owns every tensor it registers (weights, snapshot, Adam
+ *     moments) and the CUDA stream it passes to lc_create.  The library
+ *     keeps raw pointers: they must stay valid and must not move until
+ *     lc_destroy.  The library owns its own tables, staging ring, per-layer
+ *     state, pinned result block and the stores it creates.
+ *   - Work is enqueued on the context's stream in call order.  The caller
+ *     must not modify a registered tensor between lc_measure and the end of
+ *     that step's lc_pack_* / lc_commit_snapshot work on the stream (record
+ *     an event on the stream and make the training stream wait on it).
+ *   - A context is not thread-safe; use one context per thread or lock.
+ *   - Call order per context (LC_ERR_STATE otherwise):
+ *       lc_register_layout once, then per step
+ *       lc_measure -> [all-reduce of lc_layer_sums_device] -> lc_select
+ *         -> (lc_pack_device | lc_pack_async) -> lc_commit_snapshot
+ *     A step in which lc_select selected nothing may go straight to the next
+ *     lc_measure.  lc_restore may be called whenever no step is open.
+ */
+#ifndef LAYERCHECK_H
+#define LAYERCHECK_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    LC_OK = 0,
+    LC_ERR_INVALID_ARG = 1,  /* an argument is out of range or inconsistent   */
+    LC_ERR_STATE = 2,        /* the call is out of order for this context     */
+    LC_ERR_CUDA = 3,         /* a CUDA runtime call or kernel launch failed   */
+    LC_ERR_OOM = 4,          /* device or pinned host allocation failed       */
+    LC_ERR_CAPACITY = 5,     /* a destination or store is too small           */
+    LC_ERR_TIMEOUT = 6,      /* a bounded host wait on the GPU ran out        */
+    LC_ERR_NOT_FOUND = 7     /* no persisted version satisfies the request    */
+} lc_status;
+
+typedef enum { LC_BF16 = 0, LC_F32 = 1 } lc_dtype;
+
+/* How the reference weights R of Eq. 1 are kept.
+ * LC_DRIFT_SNAPSHOT  : R is the layer's weights at its last persistence, so
+ *                      u_l is the drift accumulated since then and is used
+ *                      directly as the accumulator (Eq. 2 measured end to
+ *                      end); lc_commit_snapshot refreshes R for persisted
+ *                      layers only.
+ * LC_DRIFT_ACCUMULATE: R is W(t-1) (Eq. 1 literally); lc_measure also writes
+ *                      R <- W for every layer and Eq. 2 sums u_l over steps. */
+typedef enum { LC_DRIFT_SNAPSHOT = 0, LC_DRIFT_ACCUMULATE = 1 } lc_drift_mode;
+
+/* One parameter tensor ("segment") of a layer (§2.2: embed_tokens, each
+ * transformer block, the final norm and lm_head are the layers; a layer
+ * may hold several tensors).
+ *   layer      : layer id in [0, nlayers)
+ *   w_dtype    : lc_dtype of w and snap
+ *   w          : device, numel elements, current weights W_l(t); must be
+ *                aligned to its element size (written only by lc_restore)
+ *   snap       : device, numel elements of w_dtype, the reference weights R
+ *                (written by commit / accumulate mode / restore)
+ *   exp_avg    : device, numel fp32 Adam first moment, or NULL
+ *   exp_avg_sq : device, numel fp32 Adam second moment; NULL iff exp_avg is
+ *   numel      : > 0
+ * Segments must not overlap one another. */
+typedef struct {
+    int32_t layer;
+    int32_t w_dtype;
+    void* w;
+    void* snap;
+    float* exp_avg;
+    float* exp_avg_sq;
+    int64_t numel;
+} lc_segment;
+
+typedef struct {
+    double eps_w;            /* Eq. 1 stabiliser epsilon_w (default 1e-8)        */
+    int32_t mode;            /* lc_drift_mode (default LC_DRIFT_SNAPSHOT)         */
+    int32_t pack_align;      /* section alignment of the packed layout, a power
+                                of two >= 16 (default 256)                        */
+    int32_t fuse_commit;     /* 1: lc_pack_* also writes snap <- w for the packed
+                                weights, and lc_commit_snapshot launches nothing
+                                (default 1)                                       */
+    int32_t timeout_ms;      /* bound of every host wait (default 60000)          */
+    uint64_t staging_bytes;  /* device staging ring used by lc_pack_async and
+                                lc_restore, split in two slots (default 512 MiB) */
+} lc_config;
+
+typedef struct lc_ctx lc_ctx;
+typedef struct lc_store lc_store;
+
+/* Outcome of the last lc_select (§3.3 staleness statistics included). */
+typedef struct {
+    int64_t step;                /* the step passed to lc_measure               */
+    int32_t n_selected;          /* layers persisted at this step               */
+    int32_t n_nonfinite;         /* layers whose accumulated drift was not finite
+                                    (selected; conservative counting)          */
+    uint64_t bytes;              /* packed stream size of the selected layers   */
+    int64_t max_staleness;       /* max_l (t - t_l) after this step             */
+    double weighted_staleness;   /* sum_l n_l (t - t_l) / sum_l n_l after it    */
+} lc_select_info;
+
+/* One persisted layer version in a store (the per-layer persistence
+ * history of §3.5, "metadata-driven reconstruction"). */
+typedef struct {
+    int32_t layer;
+    int32_t durable;         /* 1 once its device->host copy is known complete */
+    int64_t step;            /* t_l of this version                            */
+    const void* host_ptr;    /* packed layer block in the store (pinned host)  */
+    uint64_t bytes;          /* block size; equals lc_layer_block_bytes(layer) */
+} lc_version;
+
+/* Counters of work the context has enqueued (monotone). */
+typedef struct {
+    int64_t kernel_launches;     /* every kernel this library launched          */
+    int64_t measure_launches;
+    int64_t select_launches;
+    int64_t copy_launches;       /* pack / commit / restore copy kernels        */
+    uint64_t d2h_bytes;          /* bytes copied device -> host by the library  */
+    uint64_t h2d_bytes;          /* bytes copied host -> device by the library  */
+} lc_counters;
+
+/* Fills cfg with the defaults listed in lc_config. */
+void lc_config_default(lc_config* cfg);
+
+/* Message of the last failing call on this thread ("" if none). */
+const char* lc_last_error(void);
+
+/* Creates a context on CUDA device `device` that enqueues its work on
+ * `cuda_stream` (a cudaStream_t; NULL = the legacy default stream).  The
+ * stream stays owned by the caller.  cfg may be NULL (defaults).
+ * Errors: INVALID_ARG (bad device or config), CUDA, OOM. */
+lc_status lc_create(lc_ctx** out, int device, void* cuda_stream, const lc_config* cfg);
+
+/* Waits (bounded) for the context's work and frees everything it owns. */
+void lc_destroy(lc_ctx* ctx);
+
+/* Registers the layer -> tensor segment table, once per context (§2.2
+ * layer partition; §3.4.1 layer-aligned optimizer state).  segs: host
+ * array of nseg entries; every layer in [0, nlayers) needs >= 1 segment.
+ * A layer's segments keep their registration order in every sum and in
+ * the packed layout.  tau_mult: host array of nlayers finite factors >= 0
+ * applied to tau per layer (e.g. 10 for embeddings, §3.4.3), or NULL (1).
+ * Resets the accumulators Delta_l = 0 and last-persistence steps t_l = 0:
+ * the registered weights and snapshot are the base state of step 0.
+ * Errors: INVALID_ARG (layout, pointers not device memory, misaligned
+ * element pointers), STATE (already registered), OOM, CUDA. */
+lc_status lc_register_layout(lc_ctx* ctx, const lc_segment* segs, int32_t nseg,
+                             int32_t nlayers, const double* tau_mult);
+
+/* §3.2 Eq. 1: enqueues the segmented reduction sum|W - R|, sum|R| and the
+ * element count per layer (fp32 partial sums of at most 32 terms, combined
+ * in fp64 in a fixed order: deterministic for a given layout and device).
+ * In LC_DRIFT_ACCUMULATE mode also writes R <- W for every segment.
+ * step: the checkpoint opportunity t, strictly greater than the previous
+ * step (>= 0 for the first).  Asynchronous.
+ * Errors: STATE (not registered, or a step is open), INVALID_ARG, CUDA. */
+lc_status lc_measure(lc_ctx* ctx, int64_t step);
+
+/* Device pointer to 3*nlayers fp64 values (D_l, A_l, n_l) per layer, valid
+ * after lc_measure in stream order.  A data-parallel caller that shards
+ * every layer across ranks all-reduces (sums) this array in place on the
+ * context's stream before lc_select, so every rank takes the same
+ * decision.  Errors: STATE (not registered). */
+lc_status lc_layer_sums_device(lc_ctx* ctx, double** sums_dev);
+
+/* Makes the context keep the per-layer sums in a caller-owned device buffer
+ * of 3*nlayers fp64 (8-byte aligned) instead of its own, e.g. a tensor the
+ * caller all-reduces with its collective library.  The buffer must stay
+ * valid until lc_destroy or the next call.  Errors: STATE (not registered,
+ * or a step is open), INVALID_ARG (NULL, misaligned or not device memory). */
+lc_status lc_set_layer_sums_buffer(lc_ctx* ctx, double* sums_dev);
+
+/* §3.2 Eq. 2-4 and §3.3: on the device, u_l from the sums, the accumulator
+ * update, persist if Delta_l >= tau * tau_mult[l] or t - t_l >= max_staleness
+ * or the drift is not finite, then Delta_l <- 0, t_l <- t for the persisted
+ * layers; lays out the packed stream (selected layers ascending).  Blocks
+ * until the decision is in host memory (bounded by timeout_ms).
+ * tau: finite threshold K(t) already scaled by the learning-rate schedule.
+ * max_staleness: S_max >= 0 (0 persists every layer every step).
+ * mask_out (nlayers bytes, 1 = persist), u_out (nlayers fp64), bytes_out:
+ * host, each may be NULL.
+ * Errors: STATE (no lc_measure since the last select), INVALID_ARG,
+ * TIMEOUT, CUDA. */
+lc_status lc_select(lc_ctx* ctx, double tau, int32_t max_staleness,
+                    uint8_t* mask_out, double* u_out, uint64_t* bytes_out);
+
+/* Statistics of the last lc_select.  Errors: STATE (none yet). */
+lc_status lc_last_select_info(const lc_ctx* ctx, lc_select_info* out);
+
+/* Host array of nlayers: byte offset of each selected layer's block in the
+ * packed stream of the last lc_select (0 for unselected layers). */
+lc_status lc_last_select_offsets(const lc_ctx* ctx, uint64_t* offsets_out);
+
+/* §3.1 full layer state: gathers the selected layers' weights, exp_avg and
+ * exp_avg_sq into dst (device, 16-byte aligned, dst_capacity bytes).
+ * Layout: selected layers ascending by id; per layer every segment's W
+ * bytes, then every segment's exp_avg, then every exp_avg_sq, each section
+ * starting at a multiple of pack_align and zero-padded.  Asynchronous.
+ * With fuse_commit also writes snap <- w for those layers.
+ * Errors: STATE (no select), INVALID_ARG, CAPACITY (bytes > capacity), CUDA. */
+lc_status lc_pack_device(lc_ctx* ctx, void* dst, uint64_t dst_capacity);
+
+/* Same packed stream, through the device staging ring into `store` in
+ * pinned host memory (device->host copies on the library's copy stream).
+ * Records one pending version per selected layer; they become durable in
+ * lc_wait_durable (a step that persisted nothing is durable at once).
+ * Asynchronous.  Errors: STATE (no select, or the store
+ * still holds a pending version of a layer it would overwrite),
+ * INVALID_ARG (store built for another layout), CAPACITY, CUDA. */
+lc_status lc_pack_async(lc_ctx* ctx, lc_store* store);
+
+/* Snapshot mode: enqueues snap <- w for the layers persisted this step
+ * (Eq. 4 resets the drift reference with the accumulator); a no-op launch-
+ * wise with fuse_commit or in accumulate mode.  Closes the step.
+ * Errors: STATE (persisted layers were not packed). */
+lc_status lc_commit_snapshot(lc_ctx* ctx);
+
+/* Waits (polling, at most timeout_ms; <= 0 uses the config's) until the
+ * device->host copies of `step` issued by lc_pack_async have completed and
+ * marks those versions durable ("successfully persisted", §3.1).
+ * Errors: NOT_FOUND (no pending pack of that step), TIMEOUT, CUDA. */
+lc_status lc_wait_durable(lc_ctx* ctx, int64_t step, int32_t timeout_ms);
+
+/* §3.5 / Eq. 8: for every layer, the durable version in `store` with the
+ * largest step <= t_fail; copies those blocks host->device and scatters
+ * them into w, exp_avg, exp_avg_sq and snap (snap <- the restored w).  Sets
+ * t_l to each version's step and Delta_l = 0.  Blocks until done.
+ * layer_steps_out: host, nlayers, the chosen steps (nullable).
+ * Errors: NOT_FOUND (some layer has no version <= t_fail), STATE,
+ * INVALID_ARG, TIMEOUT, CUDA. */
+lc_status lc_restore(lc_ctx* ctx, lc_store* store, int64_t t_fail, int64_t* layer_steps_out);
+
+/* Size of one packed layer block (host-side layout query, §3.1). */
+lc_status lc_layer_block_bytes(const lc_ctx* ctx, int32_t layer, uint64_t* out);
+
+/* Library-side work counters of the context. */
+lc_status lc_get_counters(const lc_ctx* ctx, lc_counters* out);
+
+/* --- persisted-version store (pinned host memory) ---------------------- */
+
+/* Creates a store for the layout registered in ctx.
+ * versions_per_layer = 0: an append-only log of every version in one
+ *   pinned arena of capacity_bytes (every restore point stays available
+ *   until lc_store_clear).
+ * versions_per_layer = V >= 2: each layer owns V block slots and keeps its
+ *   V newest versions; capacity_bytes is ignored.  Restore points older
+ *   than a layer's oldest kept version are no longer available.
+ * The store is pinned with cudaHostAlloc and owned by the library.
+ * Errors: INVALID_ARG, STATE (ctx not registered), OOM. */
+lc_status lc_store_create(lc_store** out, const lc_ctx* ctx, uint64_t capacity_bytes,
+                          int32_t versions_per_layer);
+void lc_store_destroy(lc_store* store);
+
+/* Forgets every version (a log store reuses its arena from the start).
+ * Errors: STATE (a pending version is still being copied). */
+lc_status lc_store_clear(lc_store* store);
+
+int64_t lc_store_num_versions(const lc_store* store);
+lc_status lc_store_get_version(const lc_store* store, int64_t index, lc_version* out);
+
+/* §3.5 reconstruction plan: pick_out[l] = index of the durable version of
+ * layer l with the largest step <= t_fail (the newer record on a tie), or
+ * -1.  Returns NOT_FOUND if some layer has none. */
+lc_status lc_store_plan(const lc_store* store, int64_t t_fail, int64_t* pick_out);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* LAYERCHECK_H */

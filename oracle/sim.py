@@ -86,6 +86,7 @@ class OracleRun:
         mask, nsel, nonfinite = O.select_step(u, self.delta, self.t_last, tau, max_staleness, t,
                                               self.mode, self.tau_mult)
         self._undo = (acc_before, tl_before, np.asarray(u, dtype=np.float64).copy(), t)
+        self.last_mask = mask
         return mask
 
     def adopt_decision(self, l, persist):

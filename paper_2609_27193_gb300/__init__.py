@@ -1,0 +1,228 @@
+"""GB300-native LayerCheck hot path: Python binding of liblayercheck.so.
+
+LayerCheck (adaptive layer-wise checkpointing) measures at every checkpoint
+opportunity how far each layer's weights drifted (§3.2 Eq. 1), persists the
+layers whose accumulated drift reached a threshold or whose staleness
+reached S_max (§3.2 Eq. 2-4, §3.3) together with their Adam moments (§3.1),
+and restores the mixed-timestamp composite of the latest persisted versions
+(§3.5, Eq. 8).  Every step runs in the CUDA kernels of liblayercheck.so;
+this module only marshals torch tensors, streams and numpy arrays into the
+C ABI of include/layercheck.h (the raw functions keep their C names in
+``paper_2609_27193_gb300._abi``).  There is no CPU fallback.
+"""
+import ctypes as C
+
+import numpy as np
+
+from . import _abi
+from ._abi import (LC_BF16, LC_DRIFT_ACCUMULATE, LC_DRIFT_SNAPSHOT, LC_F32, LCError, check,
+                   lc_config, lc_counters, lc_segment, lc_select_info, lc_version)
+
+__all__ = ["LayerCheck", "Store", "LCError", "LC_BF16", "LC_F32", "LC_DRIFT_SNAPSHOT",
+           "LC_DRIFT_ACCUMULATE", "library", "segment"]
+
+
+def library():
+    """The loaded ctypes library (raises ImportError when not built)."""
+    return _abi.load()
+
+
+def _dtype_code(t):
+    import torch
+    if t.dtype == torch.bfloat16:
+        return LC_BF16
+    if t.dtype == torch.float32:
+        return LC_F32
+    raise TypeError("weights must be bfloat16 or float32, got %s" % t.dtype)
+
+
+def segment(layer, w, snap, exp_avg=None, exp_avg_sq=None):
+    """An lc_segment over torch CUDA tensors (contiguous, same numel)."""
+    for name, t in (("w", w), ("snap", snap), ("exp_avg", exp_avg), ("exp_avg_sq", exp_avg_sq)):
+        if t is not None and not t.is_contiguous():
+            raise ValueError("%s must be contiguous" % name)
+    if snap.dtype != w.dtype or snap.numel() != w.numel():
+        raise ValueError("snap must match w in dtype and size")
+    return lc_segment(int(layer), _dtype_code(w), w.data_ptr(), snap.data_ptr(),
+                      exp_avg.data_ptr() if exp_avg is not None else None,
+                      exp_avg_sq.data_ptr() if exp_avg_sq is not None else None,
+                      int(w.numel()))
+
+
+class LayerCheck:
+    """One library context on one device and one CUDA stream."""
+
+    def __init__(self, device=0, stream=None, eps_w=1e-8, mode=LC_DRIFT_SNAPSHOT,
+                 pack_align=256, fuse_commit=True, timeout_ms=60000, staging_bytes=512 << 20):
+        lib = library()
+        cfg = lc_config()
+        lib.lc_config_default(C.byref(cfg))
+        cfg.eps_w, cfg.mode, cfg.pack_align = float(eps_w), int(mode), int(pack_align)
+        cfg.fuse_commit, cfg.timeout_ms = int(bool(fuse_commit)), int(timeout_ms)
+        cfg.staging_bytes = int(staging_bytes)
+        if stream is None:
+            import torch
+            stream = torch.cuda.current_stream(device)
+        self.stream = stream
+        handle = stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream or 0)
+        ctx = C.c_void_p()
+        check(lib.lc_create(C.byref(ctx), int(device), C.c_void_p(handle), C.byref(cfg)))
+        self._lib, self._ctx = lib, ctx
+        self.device = int(device)
+        self.nlayers = 0
+        self._keep = []
+
+    # -- lifecycle -----------------------------------------------------
+    def close(self):
+        if getattr(self, "_ctx", None) and self._ctx.value:
+            self._lib.lc_destroy(self._ctx)
+            self._ctx = C.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    @property
+    def handle(self):
+        return self._ctx
+
+    # -- the path ------------------------------------------------------
+    def register_layout(self, segments, nlayers, tau_mult=None):
+        arr = (lc_segment * len(segments))(*segments)
+        mult = None
+        if tau_mult is not None:
+            m = np.ascontiguousarray(tau_mult, dtype=np.float64)
+            mult = m.ctypes.data_as(C.POINTER(C.c_double))
+            self._keep.append(m)
+        check(self._lib.lc_register_layout(self._ctx, arr, len(segments), int(nlayers), mult))
+        self.nlayers = int(nlayers)
+
+    def measure(self, step):
+        check(self._lib.lc_measure(self._ctx, int(step)))
+
+    def layer_sums_ptr(self):
+        p = C.c_void_p()
+        check(self._lib.lc_layer_sums_device(self._ctx, C.byref(p)))
+        return p.value
+
+    def set_layer_sums_buffer(self, tensor):
+        """Keep the (D, A, n) sums in a caller-owned float64 CUDA tensor of
+        3*nlayers elements (all-reduce it between measure and select)."""
+        import torch
+        if tensor.dtype != torch.float64 or tensor.numel() != 3 * self.nlayers or not tensor.is_cuda:
+            raise ValueError("need a float64 CUDA tensor of 3*nlayers elements")
+        self._keep.append(tensor)
+        check(self._lib.lc_set_layer_sums_buffer(self._ctx, C.c_void_p(tensor.data_ptr())))
+
+    def select(self, tau, max_staleness):
+        """Decision of this step: (mask uint8[N], u float64[N], packed bytes)."""
+        mask = np.zeros(self.nlayers, dtype=np.uint8)
+        u = np.zeros(self.nlayers, dtype=np.float64)
+        nbytes = C.c_uint64(0)
+        check(self._lib.lc_select(self._ctx, float(tau), int(max_staleness), mask.ctypes.data,
+                                  u.ctypes.data, C.byref(nbytes)))
+        return mask, u, nbytes.value
+
+    def info(self):
+        i = lc_select_info()
+        check(self._lib.lc_last_select_info(self._ctx, C.byref(i)))
+        return dict(step=i.step, n_selected=i.n_selected, n_nonfinite=i.n_nonfinite,
+                    bytes=i.bytes, max_staleness=i.max_staleness,
+                    weighted_staleness=i.weighted_staleness)
+
+    def offsets(self):
+        o = np.zeros(self.nlayers, dtype=np.uint64)
+        check(self._lib.lc_last_select_offsets(self._ctx, o.ctypes.data))
+        return o
+
+    def pack_device(self, dst):
+        """Gather into a uint8 CUDA (or pinned host) tensor."""
+        check(self._lib.lc_pack_device(self._ctx, C.c_void_p(dst.data_ptr()),
+                                       int(dst.numel() * dst.element_size())))
+
+    def pack_async(self, store):
+        check(self._lib.lc_pack_async(self._ctx, store.handle))
+
+    def commit_snapshot(self):
+        check(self._lib.lc_commit_snapshot(self._ctx))
+
+    def wait_durable(self, step, timeout_ms=0):
+        check(self._lib.lc_wait_durable(self._ctx, int(step), int(timeout_ms)))
+
+    def restore(self, store, t_fail):
+        steps = np.zeros(self.nlayers, dtype=np.int64)
+        check(self._lib.lc_restore(self._ctx, store.handle, int(t_fail), steps.ctypes.data))
+        return steps
+
+    def layer_block_bytes(self, layer):
+        b = C.c_uint64(0)
+        check(self._lib.lc_layer_block_bytes(self._ctx, int(layer), C.byref(b)))
+        return b.value
+
+    def counters(self):
+        c = lc_counters()
+        check(self._lib.lc_get_counters(self._ctx, C.byref(c)))
+        return {name: getattr(c, name) for name, _ in lc_counters._fields_}
+
+
+class Store:
+    """Pinned-host store of persisted layer versions (library-owned memory)."""
+
+    def __init__(self, lc, capacity_bytes=0, versions_per_layer=0):
+        self._lib = library()
+        h = C.c_void_p()
+        check(self._lib.lc_store_create(C.byref(h), lc.handle, int(capacity_bytes),
+                                        int(versions_per_layer)))
+        self._h = h
+        self.nlayers = lc.nlayers
+
+    @property
+    def handle(self):
+        return self._h
+
+    def close(self):
+        if getattr(self, "_h", None) and self._h.value:
+            self._lib.lc_store_destroy(self._h)
+            self._h = C.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def clear(self):
+        check(self._lib.lc_store_clear(self._h))
+
+    def __len__(self):
+        return int(self._lib.lc_store_num_versions(self._h))
+
+    def version(self, i):
+        v = lc_version()
+        check(self._lib.lc_store_get_version(self._h, int(i), C.byref(v)))
+        return dict(layer=v.layer, durable=bool(v.durable), step=v.step, host_ptr=v.host_ptr,
+                    bytes=v.bytes)
+
+    def versions(self):
+        return [self.version(i) for i in range(len(self))]
+
+    def block(self, i):
+        """The packed block of version i as a numpy uint8 view (no copy)."""
+        v = self.version(i)
+        if v["bytes"] == 0:
+            return np.zeros(0, np.uint8)
+        buf = (C.c_uint8 * v["bytes"]).from_address(v["host_ptr"])
+        return np.frombuffer(buf, dtype=np.uint8)
+
+    def plan(self, t_fail):
+        pick = np.zeros(self.nlayers, dtype=np.int64)
+        check(self._lib.lc_store_plan(self._h, int(t_fail), pick.ctypes.data))
+        return pick

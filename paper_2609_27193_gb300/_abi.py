@@ -1,0 +1,116 @@
+"""ctypes declarations of liblayercheck.so (include/layercheck.h).
+
+Argument marshalling only: every step of the path runs in the library's
+CUDA kernels.  Loading fails loudly when the library has not been built.
+"""
+import ctypes as C
+import os
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "liblayercheck.so")
+
+LC_OK = 0
+LC_ERR_INVALID_ARG = 1
+LC_ERR_STATE = 2
+LC_ERR_CUDA = 3
+LC_ERR_OOM = 4
+LC_ERR_CAPACITY = 5
+LC_ERR_TIMEOUT = 6
+LC_ERR_NOT_FOUND = 7
+STATUS_NAMES = {0: "LC_OK", 1: "LC_ERR_INVALID_ARG", 2: "LC_ERR_STATE", 3: "LC_ERR_CUDA",
+                4: "LC_ERR_OOM", 5: "LC_ERR_CAPACITY", 6: "LC_ERR_TIMEOUT", 7: "LC_ERR_NOT_FOUND"}
+
+LC_BF16, LC_F32 = 0, 1
+LC_DRIFT_SNAPSHOT, LC_DRIFT_ACCUMULATE = 0, 1
+
+
+class lc_segment(C.Structure):
+    _fields_ = [("layer", C.c_int32), ("w_dtype", C.c_int32), ("w", C.c_void_p),
+                ("snap", C.c_void_p), ("exp_avg", C.c_void_p), ("exp_avg_sq", C.c_void_p),
+                ("numel", C.c_int64)]
+
+
+class lc_config(C.Structure):
+    _fields_ = [("eps_w", C.c_double), ("mode", C.c_int32), ("pack_align", C.c_int32),
+                ("fuse_commit", C.c_int32), ("timeout_ms", C.c_int32),
+                ("staging_bytes", C.c_uint64)]
+
+
+class lc_select_info(C.Structure):
+    _fields_ = [("step", C.c_int64), ("n_selected", C.c_int32), ("n_nonfinite", C.c_int32),
+                ("bytes", C.c_uint64), ("max_staleness", C.c_int64),
+                ("weighted_staleness", C.c_double)]
+
+
+class lc_version(C.Structure):
+    _fields_ = [("layer", C.c_int32), ("durable", C.c_int32), ("step", C.c_int64),
+                ("host_ptr", C.c_void_p), ("bytes", C.c_uint64)]
+
+
+class lc_counters(C.Structure):
+    _fields_ = [("kernel_launches", C.c_int64), ("measure_launches", C.c_int64),
+                ("select_launches", C.c_int64), ("copy_launches", C.c_int64),
+                ("d2h_bytes", C.c_uint64), ("h2d_bytes", C.c_uint64)]
+
+
+ctx_p = C.c_void_p
+store_p = C.c_void_p
+P = C.POINTER
+
+# name -> (restype, argtypes)
+SIGNATURES = {
+    "lc_config_default": (None, [P(lc_config)]),
+    "lc_last_error": (C.c_char_p, []),
+    "lc_create": (C.c_int, [P(ctx_p), C.c_int, C.c_void_p, P(lc_config)]),
+    "lc_destroy": (None, [ctx_p]),
+    "lc_register_layout": (C.c_int, [ctx_p, P(lc_segment), C.c_int32, C.c_int32, P(C.c_double)]),
+    "lc_measure": (C.c_int, [ctx_p, C.c_int64]),
+    "lc_layer_sums_device": (C.c_int, [ctx_p, P(C.c_void_p)]),
+    "lc_set_layer_sums_buffer": (C.c_int, [ctx_p, C.c_void_p]),
+    "lc_select": (C.c_int, [ctx_p, C.c_double, C.c_int32, C.c_void_p, C.c_void_p, P(C.c_uint64)]),
+    "lc_last_select_info": (C.c_int, [ctx_p, P(lc_select_info)]),
+    "lc_last_select_offsets": (C.c_int, [ctx_p, C.c_void_p]),
+    "lc_pack_device": (C.c_int, [ctx_p, C.c_void_p, C.c_uint64]),
+    "lc_pack_async": (C.c_int, [ctx_p, store_p]),
+    "lc_commit_snapshot": (C.c_int, [ctx_p]),
+    "lc_wait_durable": (C.c_int, [ctx_p, C.c_int64, C.c_int32]),
+    "lc_restore": (C.c_int, [ctx_p, store_p, C.c_int64, C.c_void_p]),
+    "lc_layer_block_bytes": (C.c_int, [ctx_p, C.c_int32, P(C.c_uint64)]),
+    "lc_get_counters": (C.c_int, [ctx_p, P(lc_counters)]),
+    "lc_store_create": (C.c_int, [P(store_p), ctx_p, C.c_uint64, C.c_int32]),
+    "lc_store_destroy": (None, [store_p]),
+    "lc_store_clear": (C.c_int, [store_p]),
+    "lc_store_num_versions": (C.c_int64, [store_p]),
+    "lc_store_get_version": (C.c_int, [store_p, C.c_int64, P(lc_version)]),
+    "lc_store_plan": (C.c_int, [store_p, C.c_int64, C.c_void_p]),
+}
+
+_lib = None
+
+
+def load():
+    """The loaded library; raises if it was never built (no fallback)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise ImportError("liblayercheck.so is not built (run __graft_entry__.build() or "
+                              "python paper_2609_27193_gb300/build.py); there is no CPU fallback")
+        lib = C.CDLL(LIB_PATH)
+        for name, (res, args) in SIGNATURES.items():
+            fn = getattr(lib, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = lib
+    return _lib
+
+
+class LCError(RuntimeError):
+    def __init__(self, status, msg):
+        super().__init__("%s: %s" % (STATUS_NAMES.get(status, status), msg))
+        self.status = status
+
+
+def check(status):
+    if status != LC_OK:
+        raise LCError(status, load().lc_last_error().decode(errors="replace"))
+    return status

@@ -1,0 +1,1097 @@
+// lc_api.cu -- host side of liblayercheck.so: the C ABI of layercheck.h.
+//
+// Owns the per-context tables (measure work partition, packed-layout
+// sections), the per-layer state (Delta_l, t_l), the pinned decision block,
+// the device staging ring and the pinned-host version stores, and drives
+// the kernels of lc_measure.cu, lc_select.cu and lc_copy.cu on the caller's
+// stream.  No compute happens here: every step of the path runs on the GPU.
+#include "layercheck.h"
+#include "lc_internal.cuh"
+
+#include <algorithm>
+#include <chrono>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <set>
+#include <string>
+#include <thread>
+#include <vector>
+
+using namespace lc;
+
+// ---------------------------------------------------------------------------
+// errors
+// ---------------------------------------------------------------------------
+namespace {
+
+thread_local std::string g_err;
+
+lc_status fail(lc_status st, const char* fmt, ...) {
+    char buf[1024];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_err = buf;
+    return st;
+}
+
+#define LC_CUDA(call)                                                                   \
+    do {                                                                                \
+        cudaError_t e_ = (call);                                                        \
+        if (e_ != cudaSuccess) {                                                        \
+            cudaGetLastError();                                                         \
+            return fail(e_ == cudaErrorMemoryAllocation ? LC_ERR_OOM : LC_ERR_CUDA,     \
+                        "%s failed: %s (%s:%d)", #call, cudaGetErrorString(e_), __FILE__, \
+                        __LINE__);                                                      \
+        }                                                                               \
+    } while (0)
+
+#define LC_TRY(expr)                  \
+    do {                              \
+        lc_status st_ = (expr);       \
+        if (st_ != LC_OK) return st_; \
+    } while (0)
+
+// Restores the caller's current device on scope exit.
+struct DeviceGuard {
+    int prev = -1;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+        if (prev != dev) cudaSetDevice(dev);
+    }
+    ~DeviceGuard() {
+        int cur = -1;
+        if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+    }
+};
+
+uint64_t round_up(uint64_t x, uint64_t a) { return (x + a - 1) / a * a; }
+
+// Polls an event until it completes or timeout_ms passes.
+lc_status wait_event(cudaEvent_t ev, int timeout_ms, const char* what) {
+    using clk = std::chrono::steady_clock;
+    const auto t0 = clk::now();
+    long spins = 0;
+    for (;;) {
+        const cudaError_t q = cudaEventQuery(ev);
+        if (q == cudaSuccess) return LC_OK;
+        if (q != cudaErrorNotReady) {
+            cudaGetLastError();
+            return fail(LC_ERR_CUDA, "%s: %s", what, cudaGetErrorString(q));
+        }
+        const auto ms = std::chrono::duration_cast<std::chrono::milliseconds>(clk::now() - t0).count();
+        if (ms > timeout_ms) return fail(LC_ERR_TIMEOUT, "%s: not complete after %d ms", what, timeout_ms);
+        if (++spins > 20000) std::this_thread::sleep_for(std::chrono::microseconds(50));
+    }
+}
+
+lc_status check_device_ptr(const void* p, int device, const char* what, bool allow_host) {
+    cudaPointerAttributes a;
+    const cudaError_t e = cudaPointerGetAttributes(&a, p);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return fail(LC_ERR_INVALID_ARG, "%s: not a CUDA-visible pointer (%s)", what, cudaGetErrorString(e));
+    }
+    if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) {
+        if (a.type == cudaMemoryTypeDevice && a.device != device)
+            return fail(LC_ERR_INVALID_ARG, "%s: memory of device %d, context is on device %d", what,
+                        a.device, device);
+        return LC_OK;
+    }
+    if (allow_host && a.type == cudaMemoryTypeHost) return LC_OK;
+    return fail(LC_ERR_INVALID_ARG, "%s: not device memory", what);
+}
+
+std::mutex g_store_mu;
+std::set<const lc_store*> g_live_stores;
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// objects
+// ---------------------------------------------------------------------------
+struct StoreVersion {
+    int64_t id;
+    int32_t layer;
+    int32_t durable;
+    int64_t step;
+    uint64_t off;      // byte offset in the arena
+    uint64_t bytes;
+    int32_t slot;      // ring slot (ring mode) or -1
+};
+
+struct lc_store {
+    int32_t nlayers = 0;
+    int32_t per_layer = 0;                 // 0 = log
+    uint64_t capacity = 0;
+    uint8_t* arena = nullptr;
+    uint64_t top = 0;                      // log mode
+    std::vector<uint64_t> layer_bytes;
+    std::vector<uint64_t> layer_base;      // ring mode
+    std::vector<int64_t> layer_writes;     // ring mode: versions ever written
+    std::vector<StoreVersion> versions;
+    int64_t next_id = 0;
+    std::vector<cudaEvent_t> inflight;     // copies still writing into the arena
+};
+
+struct PendingPack {
+    int64_t step;
+    cudaEvent_t done;
+    lc_store* store;
+    std::vector<int64_t> ids;
+};
+
+enum State { kNew = 0, kReady, kMeasured, kSelected, kPacked };
+
+struct lc_ctx {
+    int device = 0;
+    cudaStream_t stream = nullptr;
+    cudaStream_t copy_stream = nullptr;
+    lc_config cfg{};
+    int sms = 0;
+    State state = kNew;
+    int64_t last_step = -1;
+
+    int32_t nseg = 0, nlayers = 0;
+    std::vector<lc_segment> segs;          // measure order
+    std::vector<int32_t> layer_seg_begin;  // [nlayers+1]
+    std::vector<int64_t> layer_numel;
+    std::vector<uint64_t> layer_bytes;
+    std::vector<SectionDev> secs;          // packed order, layer-major
+    std::vector<int32_t> layer_sec_begin;  // [nlayers+1]
+    std::vector<int32_t> sec_seg;          // segment (measure order) of each section
+    std::vector<int32_t> sec_part;         // 0 = W, 1 = exp_avg, 2 = exp_avg_sq
+    int measure_grid = 0, copy_grid = 0, nslots = 0;
+    bool any_write_ref = false;
+
+    // device memory
+    void* d_tables = nullptr;
+    MeasureParams mp{};
+    SelectParams sp{};
+    CopyDesc* d_pack_desc = nullptr;
+    CopyDesc* d_commit_desc = nullptr;
+    CopyDesc* d_restore_desc = nullptr;
+    uint8_t* d_result = nullptr;
+    uint8_t* h_result = nullptr;           // pinned
+    ResultLayout rl{};
+    cudaEvent_t ev_result = nullptr;
+
+    // staging ring
+    uint8_t* d_staging = nullptr;
+    uint64_t slot_bytes = 0;
+    cudaEvent_t ev_slot_free[2] = {nullptr, nullptr};
+    cudaEvent_t ev_slot_filled[2] = {nullptr, nullptr};
+    bool slot_busy[2] = {false, false};
+
+    // last decision
+    bool have_select = false;
+    ResultHeader hdr{};
+    std::vector<uint8_t> mask;
+    std::vector<uint64_t> offsets;
+    std::vector<PendingPack> pending;
+    lc_counters counters{};
+};
+
+// ---------------------------------------------------------------------------
+// config, errors, create, destroy
+// ---------------------------------------------------------------------------
+extern "C" void lc_config_default(lc_config* cfg) {
+    if (!cfg) return;
+    std::memset(cfg, 0, sizeof *cfg);
+    cfg->eps_w = 1e-8;
+    cfg->mode = LC_DRIFT_SNAPSHOT;
+    cfg->pack_align = 256;
+    cfg->fuse_commit = 1;
+    cfg->timeout_ms = 60000;
+    cfg->staging_bytes = 512ull << 20;
+}
+
+extern "C" const char* lc_last_error(void) { return g_err.c_str(); }
+
+extern "C" lc_status lc_create(lc_ctx** out, int device, void* cuda_stream, const lc_config* cfg) {
+    g_err.clear();
+    if (!out) return fail(LC_ERR_INVALID_ARG, "lc_create: out is NULL");
+    *out = nullptr;
+    lc_config c;
+    if (cfg) c = *cfg;
+    else lc_config_default(&c);
+    if (!(c.eps_w >= 0.0) || !std::isfinite(c.eps_w))
+        return fail(LC_ERR_INVALID_ARG, "lc_create: eps_w must be finite and >= 0");
+    if (c.mode != LC_DRIFT_SNAPSHOT && c.mode != LC_DRIFT_ACCUMULATE)
+        return fail(LC_ERR_INVALID_ARG, "lc_create: unknown drift mode %d", c.mode);
+    if (c.pack_align < 16 || (c.pack_align & (c.pack_align - 1)))
+        return fail(LC_ERR_INVALID_ARG, "lc_create: pack_align must be a power of two >= 16");
+    if (c.timeout_ms <= 0) return fail(LC_ERR_INVALID_ARG, "lc_create: timeout_ms must be > 0");
+    if (c.staging_bytes < (2u << 20))
+        return fail(LC_ERR_INVALID_ARG, "lc_create: staging_bytes must be >= 2 MiB");
+    int ndev = 0;
+    LC_CUDA(cudaGetDeviceCount(&ndev));
+    if (device < 0 || device >= ndev)
+        return fail(LC_ERR_INVALID_ARG, "lc_create: device %d out of range (%d devices)", device, ndev);
+    cudaDeviceProp prop;
+    LC_CUDA(cudaGetDeviceProperties(&prop, device));
+    if (prop.major * 10 + prop.minor != 103)
+        return fail(LC_ERR_INVALID_ARG,
+                    "lc_create: liblayercheck is built for sm_103a only; device %d is sm_%d%d", device,
+                    prop.major, prop.minor);
+    DeviceGuard g(device);
+    lc_ctx* ctx = new lc_ctx();
+    ctx->device = device;
+    ctx->stream = static_cast<cudaStream_t>(cuda_stream);
+    ctx->cfg = c;
+    ctx->sms = prop.multiProcessorCount;
+    cudaError_t e = cudaStreamCreateWithFlags(&ctx->copy_stream, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->ev_result, cudaEventDisableTiming);
+    for (int i = 0; i < 2 && e == cudaSuccess; ++i) {
+        e = cudaEventCreateWithFlags(&ctx->ev_slot_free[i], cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->ev_slot_filled[i], cudaEventDisableTiming);
+    }
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        lc_destroy(ctx);
+        return fail(LC_ERR_CUDA, "lc_create: %s", cudaGetErrorString(e));
+    }
+    *out = ctx;
+    return LC_OK;
+}
+
+extern "C" void lc_destroy(lc_ctx* ctx) {
+    if (!ctx) return;
+    DeviceGuard g(ctx->device);
+    if (ctx->stream || ctx->copy_stream) {
+        cudaEvent_t ev;
+        if (cudaEventCreateWithFlags(&ev, cudaEventDisableTiming) == cudaSuccess) {
+            if (cudaEventRecord(ev, ctx->stream) == cudaSuccess) wait_event(ev, ctx->cfg.timeout_ms, "lc_destroy");
+            if (ctx->copy_stream && cudaEventRecord(ev, ctx->copy_stream) == cudaSuccess)
+                wait_event(ev, ctx->cfg.timeout_ms, "lc_destroy");
+            cudaEventDestroy(ev);
+        }
+    }
+    for (auto& pp : ctx->pending) cudaEventDestroy(pp.done);
+    cudaFree(ctx->d_tables);
+    cudaFree(ctx->d_staging);
+    if (ctx->h_result) cudaFreeHost(ctx->h_result);
+    if (ctx->ev_result) cudaEventDestroy(ctx->ev_result);
+    for (int i = 0; i < 2; ++i) {
+        if (ctx->ev_slot_free[i]) cudaEventDestroy(ctx->ev_slot_free[i]);
+        if (ctx->ev_slot_filled[i]) cudaEventDestroy(ctx->ev_slot_filled[i]);
+    }
+    if (ctx->copy_stream) cudaStreamDestroy(ctx->copy_stream);
+    cudaGetLastError();
+    delete ctx;
+}
+
+// ---------------------------------------------------------------------------
+// layout registration
+// ---------------------------------------------------------------------------
+namespace {
+
+// Bump allocator over one device allocation holding every table.
+struct TablePlan {
+    size_t size = 0;
+    size_t take(size_t bytes) {
+        size_t off = round_up(size, 256);
+        size = off + bytes;
+        return off;
+    }
+};
+
+}  // namespace
+
+extern "C" lc_status lc_register_layout(lc_ctx* ctx, const lc_segment* segs, int32_t nseg,
+                                        int32_t nlayers, const double* tau_mult) {
+    g_err.clear();
+    if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_register_layout: ctx is NULL");
+    if (ctx->state != kNew) return fail(LC_ERR_STATE, "lc_register_layout: layout already registered");
+    if (!segs || nseg <= 0) return fail(LC_ERR_INVALID_ARG, "lc_register_layout: no segments");
+    if (nlayers <= 0) return fail(LC_ERR_INVALID_ARG, "lc_register_layout: nlayers must be > 0");
+    DeviceGuard g(ctx->device);
+
+    std::vector<int32_t> per_layer(nlayers, 0);
+    for (int32_t i = 0; i < nseg; ++i) {
+        const lc_segment& s = segs[i];
+        if (s.layer < 0 || s.layer >= nlayers)
+            return fail(LC_ERR_INVALID_ARG, "segment %d: layer %d outside [0, %d)", i, s.layer, nlayers);
+        if (s.w_dtype != LC_BF16 && s.w_dtype != LC_F32)
+            return fail(LC_ERR_INVALID_ARG, "segment %d: unknown dtype %d", i, s.w_dtype);
+        if (s.numel <= 0) return fail(LC_ERR_INVALID_ARG, "segment %d: numel must be > 0", i);
+        if (!s.w || !s.snap) return fail(LC_ERR_INVALID_ARG, "segment %d: w and snap are required", i);
+        if ((s.exp_avg == nullptr) != (s.exp_avg_sq == nullptr))
+            return fail(LC_ERR_INVALID_ARG, "segment %d: exp_avg and exp_avg_sq must both be set or both NULL", i);
+        const uintptr_t esz = s.w_dtype == LC_BF16 ? 2 : 4;
+        if ((uintptr_t(s.w) % esz) || (uintptr_t(s.snap) % esz))
+            return fail(LC_ERR_INVALID_ARG, "segment %d: w/snap not aligned to the element size", i);
+        if (s.exp_avg && ((uintptr_t(s.exp_avg) % 4) || (uintptr_t(s.exp_avg_sq) % 4)))
+            return fail(LC_ERR_INVALID_ARG, "segment %d: Adam moments not 4-byte aligned", i);
+        char what[64];
+        snprintf(what, sizeof what, "segment %d w", i);
+        LC_TRY(check_device_ptr(s.w, ctx->device, what, false));
+        snprintf(what, sizeof what, "segment %d snap", i);
+        LC_TRY(check_device_ptr(s.snap, ctx->device, what, false));
+        if (s.exp_avg) {
+            snprintf(what, sizeof what, "segment %d exp_avg", i);
+            LC_TRY(check_device_ptr(s.exp_avg, ctx->device, what, false));
+            snprintf(what, sizeof what, "segment %d exp_avg_sq", i);
+            LC_TRY(check_device_ptr(s.exp_avg_sq, ctx->device, what, false));
+        }
+        per_layer[s.layer] += 1;
+    }
+    for (int32_t l = 0; l < nlayers; ++l)
+        if (per_layer[l] == 0) return fail(LC_ERR_INVALID_ARG, "layer %d has no segment", l);
+    std::vector<double> mult(nlayers, 1.0);
+    if (tau_mult) {
+        for (int32_t l = 0; l < nlayers; ++l) {
+            if (!std::isfinite(tau_mult[l]) || tau_mult[l] < 0.0)
+                return fail(LC_ERR_INVALID_ARG, "tau_mult[%d] must be finite and >= 0", l);
+            mult[l] = tau_mult[l];
+        }
+    }
+
+    // measure order: layers ascending, registration order inside a layer
+    std::vector<int32_t> order(nseg);
+    for (int32_t i = 0; i < nseg; ++i) order[i] = i;
+    std::stable_sort(order.begin(), order.end(),
+                     [&](int32_t a, int32_t b) { return segs[a].layer < segs[b].layer; });
+    ctx->nseg = nseg;
+    ctx->nlayers = nlayers;
+    ctx->segs.resize(nseg);
+    for (int32_t i = 0; i < nseg; ++i) ctx->segs[i] = segs[order[i]];
+    ctx->layer_seg_begin.assign(nlayers + 1, 0);
+    for (int32_t i = 0; i < nseg; ++i) ctx->layer_seg_begin[ctx->segs[i].layer + 1] += 1;
+    for (int32_t l = 0; l < nlayers; ++l) ctx->layer_seg_begin[l + 1] += ctx->layer_seg_begin[l];
+
+    // measure work space: 16-byte virtual vectors
+    std::vector<SegDev> sd(nseg);
+    int64_t V = 0;
+    for (int32_t i = 0; i < nseg; ++i) {
+        const lc_segment& s = ctx->segs[i];
+        const int esz_log2 = s.w_dtype == LC_BF16 ? 1 : 2;
+        const int ve = 16 >> esz_log2;
+        SegDev& d = sd[i];
+        d.w = static_cast<const uint8_t*>(s.w);
+        d.r = static_cast<uint8_t*>(s.snap);
+        d.numel = s.numel;
+        d.lead = int32_t((uintptr_t(s.w) & 15) >> esz_log2);
+        d.esz_log2 = esz_log2;
+        d.coaligned = (uintptr_t(s.w) & 15) == (uintptr_t(s.snap) & 15);
+        d.layer = s.layer;
+        d.nvec = (int64_t(d.lead) + s.numel + ve - 1) / ve;
+        d.vec_begin = V;
+        V += d.nvec;
+    }
+    int occ = 0;
+    LC_CUDA(measure_occupancy(&occ));
+    if (occ <= 0) occ = 1;
+    const int64_t G = std::min<int64_t>(V, int64_t(ctx->sms) * occ);
+    ctx->measure_grid = int(G);
+    std::vector<int64_t> cta_vec(G + 1);
+    std::vector<int32_t> cta_seg0(G), cta_slot0(G);
+    std::vector<int32_t> seg_slot_begin(nseg + 1, -1);
+    int32_t slot = 0, s = 0;
+    for (int64_t b = 0; b <= G; ++b) cta_vec[b] = V * b / G;
+    for (int64_t b = 0; b < G; ++b) {
+        const int64_t v0 = cta_vec[b], v1 = cta_vec[b + 1];
+        while (s < nseg && sd[s].vec_begin + sd[s].nvec <= v0) ++s;
+        cta_seg0[b] = s;
+        cta_slot0[b] = slot;
+        for (int32_t t = s; t < nseg && sd[t].vec_begin < v1; ++t) {
+            if (seg_slot_begin[t] < 0) seg_slot_begin[t] = slot;
+            ++slot;
+        }
+    }
+    seg_slot_begin[nseg] = slot;
+    for (int32_t t = nseg - 1; t >= 0; --t)
+        if (seg_slot_begin[t] < 0) seg_slot_begin[t] = seg_slot_begin[t + 1];
+    ctx->nslots = slot;
+
+    // packed layout: per layer all W sections, then exp_avg, then exp_avg_sq
+    const uint64_t align = uint64_t(ctx->cfg.pack_align);
+    ctx->layer_numel.assign(nlayers, 0);
+    ctx->layer_bytes.assign(nlayers, 0);
+    ctx->layer_sec_begin.assign(nlayers + 1, 0);
+    std::vector<int32_t> wsec(nlayers, 0);
+    ctx->secs.clear();
+    ctx->sec_seg.clear();
+    ctx->sec_part.clear();
+    for (int32_t l = 0; l < nlayers; ++l) {
+        ctx->layer_sec_begin[l] = int32_t(ctx->secs.size());
+        uint64_t off = 0;
+        for (int part = 0; part < 3; ++part) {
+            for (int32_t i = ctx->layer_seg_begin[l]; i < ctx->layer_seg_begin[l + 1]; ++i) {
+                const lc_segment& sg = ctx->segs[i];
+                if (part == 0) ctx->layer_numel[l] += sg.numel;
+                const uint64_t esz = sg.w_dtype == LC_BF16 ? 2 : 4;
+                const uint64_t nbytes = part == 0 ? uint64_t(sg.numel) * esz
+                                        : (sg.exp_avg ? uint64_t(sg.numel) * 4 : 0);
+                if (nbytes == 0) continue;
+                SectionDev sec;
+                sec.off_in_layer = off;
+                sec.nbytes = nbytes;
+                sec.span = round_up(nbytes, align);
+                sec.src = part == 0 ? static_cast<const uint8_t*>(sg.w)
+                          : part == 1 ? reinterpret_cast<const uint8_t*>(sg.exp_avg)
+                                      : reinterpret_cast<const uint8_t*>(sg.exp_avg_sq);
+                sec.ref = part == 0 ? static_cast<uint8_t*>(sg.snap) : nullptr;
+                ctx->secs.push_back(sec);
+                ctx->sec_seg.push_back(i);
+                ctx->sec_part.push_back(part);
+                if (part == 0) wsec[l] += 1;
+                off += sec.span;
+            }
+        }
+        ctx->layer_bytes[l] = off;
+    }
+    ctx->layer_sec_begin[nlayers] = int32_t(ctx->secs.size());
+    const int32_t nsec = int32_t(ctx->secs.size());
+
+    int cocc = 0;
+    LC_CUDA(copy_occupancy(&cocc));
+    ctx->copy_grid = ctx->sms * std::max(1, cocc);
+
+    // one device allocation for every table and small state array
+    TablePlan tp;
+    const size_t o_segs = tp.take(sizeof(SegDev) * nseg);
+    const size_t o_ctav = tp.take(sizeof(int64_t) * (G + 1));
+    const size_t o_ctas = tp.take(sizeof(int32_t) * G);
+    const size_t o_ctal = tp.take(sizeof(int32_t) * G);
+    const size_t o_segslot = tp.take(sizeof(int32_t) * (nseg + 1));
+    const size_t o_lsb = tp.take(sizeof(int32_t) * (nlayers + 1));
+    const size_t o_part = tp.take(sizeof(double2) * std::max(1, ctx->nslots));
+    const size_t o_segsum = tp.take(sizeof(double) * 2 * nseg);
+    const size_t o_sums = tp.take(sizeof(double) * 3 * nlayers);
+    const size_t o_ticket = tp.take(sizeof(unsigned int));
+    const size_t o_delta = tp.take(sizeof(double) * nlayers);
+    const size_t o_tlast = tp.take(sizeof(int64_t) * nlayers);
+    const size_t o_mult = tp.take(sizeof(double) * nlayers);
+    const size_t o_lnumel = tp.take(sizeof(int64_t) * nlayers);
+    const size_t o_lbytes = tp.take(sizeof(uint64_t) * nlayers);
+    const size_t o_lsec = tp.take(sizeof(int32_t) * (nlayers + 1));
+    const size_t o_lwsec = tp.take(sizeof(int32_t) * nlayers);
+    const size_t o_secs = tp.take(sizeof(SectionDev) * std::max(1, nsec));
+    const size_t o_scratch = tp.take(sizeof(int64_t) * 3 * nlayers);
+    ctx->rl = result_layout(nlayers);
+    const size_t o_result = tp.take(ctx->rl.total);
+    const size_t o_pdesc = tp.take(sizeof(CopyDesc) * std::max(1, nsec));
+    const size_t o_cdesc = tp.take(sizeof(CopyDesc) * nseg);
+    const size_t o_rdesc = tp.take(sizeof(CopyDesc) * std::max(1, nsec));
+    const size_t total = tp.size;
+
+    std::vector<uint8_t> host(total, 0);
+    auto put = [&](size_t off, const void* src, size_t n) { if (n) std::memcpy(host.data() + off, src, n); };
+    put(o_segs, sd.data(), sizeof(SegDev) * nseg);
+    put(o_ctav, cta_vec.data(), sizeof(int64_t) * (G + 1));
+    put(o_ctas, cta_seg0.data(), sizeof(int32_t) * G);
+    put(o_ctal, cta_slot0.data(), sizeof(int32_t) * G);
+    put(o_segslot, seg_slot_begin.data(), sizeof(int32_t) * (nseg + 1));
+    put(o_lsb, ctx->layer_seg_begin.data(), sizeof(int32_t) * (nlayers + 1));
+    put(o_mult, mult.data(), sizeof(double) * nlayers);
+    put(o_lnumel, ctx->layer_numel.data(), sizeof(int64_t) * nlayers);
+    put(o_lbytes, ctx->layer_bytes.data(), sizeof(uint64_t) * nlayers);
+    put(o_lsec, ctx->layer_sec_begin.data(), sizeof(int32_t) * (nlayers + 1));
+    put(o_lwsec, wsec.data(), sizeof(int32_t) * nlayers);
+    put(o_secs, ctx->secs.data(), sizeof(SectionDev) * nsec);
+    // accumulators, t_l, ticket and partials start at zero (the host image is zeroed)
+
+    void* dev = nullptr;
+    LC_CUDA(cudaMalloc(&dev, total));
+    ctx->d_tables = dev;
+    LC_CUDA(cudaMemcpy(dev, host.data(), total, cudaMemcpyHostToDevice));
+    uint8_t* base = static_cast<uint8_t*>(dev);
+
+    MeasureParams& mp = ctx->mp;
+    mp.segs = reinterpret_cast<const SegDev*>(base + o_segs);
+    mp.cta_vec_begin = reinterpret_cast<const int64_t*>(base + o_ctav);
+    mp.cta_seg0 = reinterpret_cast<const int32_t*>(base + o_ctas);
+    mp.cta_slot0 = reinterpret_cast<const int32_t*>(base + o_ctal);
+    mp.seg_slot_begin = reinterpret_cast<const int32_t*>(base + o_segslot);
+    mp.layer_seg_begin = reinterpret_cast<const int32_t*>(base + o_lsb);
+    mp.partials = reinterpret_cast<double2*>(base + o_part);
+    mp.seg_sums = reinterpret_cast<double*>(base + o_segsum);
+    mp.sums = reinterpret_cast<double*>(base + o_sums);
+    mp.ticket = reinterpret_cast<unsigned int*>(base + o_ticket);
+    mp.nseg = nseg;
+    mp.nlayers = nlayers;
+
+    SelectParams& sp = ctx->sp;
+    sp.sums = mp.sums;
+    sp.delta = reinterpret_cast<double*>(base + o_delta);
+    sp.t_last = reinterpret_cast<int64_t*>(base + o_tlast);
+    sp.tau_mult = reinterpret_cast<const double*>(base + o_mult);
+    sp.layer_numel = reinterpret_cast<const int64_t*>(base + o_lnumel);
+    sp.layer_bytes = reinterpret_cast<const uint64_t*>(base + o_lbytes);
+    sp.layer_sec_begin = reinterpret_cast<const int32_t*>(base + o_lsec);
+    sp.layer_wsec_count = reinterpret_cast<const int32_t*>(base + o_lwsec);
+    sp.secs = reinterpret_cast<const SectionDev*>(base + o_secs);
+    sp.layer_scratch = reinterpret_cast<int64_t*>(base + o_scratch);
+    sp.result = base + o_result;
+    sp.pack_desc = reinterpret_cast<CopyDesc*>(base + o_pdesc);
+    sp.commit_desc = reinterpret_cast<CopyDesc*>(base + o_cdesc);
+    sp.nlayers = nlayers;
+    sp.mode = ctx->cfg.mode;
+    sp.fuse_commit = ctx->cfg.fuse_commit;
+    sp.eps_w = ctx->cfg.eps_w;
+    ctx->d_result = sp.result;
+    ctx->d_pack_desc = sp.pack_desc;
+    ctx->d_commit_desc = sp.commit_desc;
+    ctx->d_restore_desc = reinterpret_cast<CopyDesc*>(base + o_rdesc);
+
+    LC_CUDA(cudaHostAlloc(reinterpret_cast<void**>(&ctx->h_result), ctx->rl.total, cudaHostAllocDefault));
+    ctx->mask.assign(nlayers, 0);
+    ctx->offsets.assign(nlayers, 0);
+    ctx->state = kReady;
+    ctx->last_step = -1;
+    return LC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// per-step path
+// ---------------------------------------------------------------------------
+namespace {
+
+bool step_open(const lc_ctx* ctx) {
+    if (ctx->state == kMeasured || ctx->state == kPacked) return true;
+    if (ctx->state == kSelected) return ctx->hdr.n_selected > 0;
+    return false;
+}
+
+}  // namespace
+
+extern "C" lc_status lc_measure(lc_ctx* ctx, int64_t step) {
+    g_err.clear();
+    if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_measure: ctx is NULL");
+    if (ctx->state == kNew) return fail(LC_ERR_STATE, "lc_measure: no layout registered");
+    if (step_open(ctx)) return fail(LC_ERR_STATE, "lc_measure: the previous step is still open");
+    if (step < 0 || step <= ctx->last_step)
+        return fail(LC_ERR_INVALID_ARG, "lc_measure: step %lld must exceed the previous step %lld",
+                    (long long)step, (long long)ctx->last_step);
+    DeviceGuard g(ctx->device);
+    LC_CUDA(launch_measure(ctx->mp, ctx->measure_grid, ctx->cfg.mode == LC_DRIFT_ACCUMULATE, ctx->stream));
+    ctx->counters.kernel_launches += 1;
+    ctx->counters.measure_launches += 1;
+    ctx->last_step = step;
+    ctx->state = kMeasured;
+    return LC_OK;
+}
+
+extern "C" lc_status lc_layer_sums_device(lc_ctx* ctx, double** sums_dev) {
+    g_err.clear();
+    if (!ctx || !sums_dev) return fail(LC_ERR_INVALID_ARG, "lc_layer_sums_device: NULL argument");
+    if (ctx->state == kNew) return fail(LC_ERR_STATE, "lc_layer_sums_device: no layout registered");
+    *sums_dev = ctx->mp.sums;
+    return LC_OK;
+}
+
+extern "C" lc_status lc_set_layer_sums_buffer(lc_ctx* ctx, double* sums_dev) {
+    g_err.clear();
+    if (!ctx || !sums_dev) return fail(LC_ERR_INVALID_ARG, "lc_set_layer_sums_buffer: NULL argument");
+    if (ctx->state == kNew) return fail(LC_ERR_STATE, "lc_set_layer_sums_buffer: no layout registered");
+    if (step_open(ctx)) return fail(LC_ERR_STATE, "lc_set_layer_sums_buffer: a step is open");
+    if (uintptr_t(sums_dev) & 7) return fail(LC_ERR_INVALID_ARG, "lc_set_layer_sums_buffer: buffer not 8-byte aligned");
+    DeviceGuard g(ctx->device);
+    LC_TRY(check_device_ptr(sums_dev, ctx->device, "lc_set_layer_sums_buffer", false));
+    ctx->mp.sums = sums_dev;
+    ctx->sp.sums = sums_dev;
+    return LC_OK;
+}
+
+extern "C" lc_status lc_select(lc_ctx* ctx, double tau, int32_t max_staleness, uint8_t* mask_out,
+                               double* u_out, uint64_t* bytes_out) {
+    g_err.clear();
+    if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_select: ctx is NULL");
+    if (ctx->state != kMeasured) return fail(LC_ERR_STATE, "lc_select: call lc_measure first");
+    if (!std::isfinite(tau)) return fail(LC_ERR_INVALID_ARG, "lc_select: tau must be finite");
+    if (max_staleness < 0) return fail(LC_ERR_INVALID_ARG, "lc_select: max_staleness must be >= 0");
+    DeviceGuard g(ctx->device);
+    SelectParams p = ctx->sp;
+    p.tau = tau;
+    p.max_staleness = max_staleness;
+    p.step = ctx->last_step;
+    LC_CUDA(launch_select(p, ctx->stream));
+    ctx->counters.kernel_launches += 1;
+    ctx->counters.select_launches += 1;
+    LC_CUDA(cudaMemcpyAsync(ctx->h_result, ctx->d_result, ctx->rl.total, cudaMemcpyDeviceToHost, ctx->stream));
+    ctx->counters.d2h_bytes += ctx->rl.total;
+    LC_CUDA(cudaEventRecord(ctx->ev_result, ctx->stream));
+    LC_TRY(wait_event(ctx->ev_result, ctx->cfg.timeout_ms, "lc_select"));
+
+    ResultHeader h;
+    std::memcpy(&h, ctx->h_result, sizeof h);
+    if (h.magic != kResultMagic || h.step != ctx->last_step)
+        return fail(LC_ERR_CUDA, "lc_select: decision block is corrupt");
+    const uint8_t* m = ctx->h_result + ctx->rl.mask_off;
+    const double* u = reinterpret_cast<const double*>(ctx->h_result + ctx->rl.u_off);
+    const uint64_t* o = reinterpret_cast<const uint64_t*>(ctx->h_result + ctx->rl.off_off);
+    uint64_t check = 0;
+    for (int32_t l = 0; l < ctx->nlayers; ++l) {
+        ctx->mask[l] = m[l];
+        ctx->offsets[l] = o[l];
+        if (m[l]) check += ctx->layer_bytes[l];
+    }
+    if (check != h.bytes) return fail(LC_ERR_CUDA, "lc_select: decision block byte count mismatch");
+    if (mask_out) std::memcpy(mask_out, m, size_t(ctx->nlayers));
+    if (u_out) std::memcpy(u_out, u, sizeof(double) * size_t(ctx->nlayers));
+    if (bytes_out) *bytes_out = h.bytes;
+    ctx->hdr = h;
+    ctx->have_select = true;
+    ctx->state = kSelected;
+    return LC_OK;
+}
+
+extern "C" lc_status lc_last_select_info(const lc_ctx* ctx, lc_select_info* out) {
+    g_err.clear();
+    if (!ctx || !out) return fail(LC_ERR_INVALID_ARG, "lc_last_select_info: NULL argument");
+    if (!ctx->have_select) return fail(LC_ERR_STATE, "lc_last_select_info: no lc_select yet");
+    out->step = ctx->hdr.step;
+    out->n_selected = ctx->hdr.n_selected;
+    out->n_nonfinite = ctx->hdr.n_nonfinite;
+    out->bytes = ctx->hdr.bytes;
+    out->max_staleness = ctx->hdr.max_staleness;
+    out->weighted_staleness = ctx->hdr.weighted_staleness;
+    return LC_OK;
+}
+
+extern "C" lc_status lc_last_select_offsets(const lc_ctx* ctx, uint64_t* offsets_out) {
+    g_err.clear();
+    if (!ctx || !offsets_out) return fail(LC_ERR_INVALID_ARG, "lc_last_select_offsets: NULL argument");
+    if (!ctx->have_select) return fail(LC_ERR_STATE, "lc_last_select_offsets: no lc_select yet");
+    std::memcpy(offsets_out, ctx->offsets.data(), sizeof(uint64_t) * size_t(ctx->nlayers));
+    return LC_OK;
+}
+
+namespace {
+
+lc_status launch_copy_range(lc_ctx* ctx, const CopyDesc* desc, int ndesc, int mode, uint64_t lo,
+                            uint64_t hi, uint8_t* base, cudaStream_t s) {
+    if (hi <= lo || ndesc <= 0) return LC_OK;
+    CopyParams p;
+    p.desc = desc;
+    p.ndesc = ndesc;
+    p.mode = mode;
+    p.lo = lo;
+    p.hi = hi;
+    p.base = base;
+    const uint64_t units = (hi - lo) >> 4;
+    const int grid = int(std::max<uint64_t>(1, std::min<uint64_t>(uint64_t(ctx->copy_grid), units)));
+    LC_CUDA(launch_copy(p, grid, s));
+    ctx->counters.kernel_launches += 1;
+    ctx->counters.copy_launches += 1;
+    return LC_OK;
+}
+
+lc_status ensure_staging(lc_ctx* ctx) {
+    if (ctx->d_staging) return LC_OK;
+    ctx->slot_bytes = (ctx->cfg.staging_bytes / 2) & ~uint64_t(4095);
+    void* p = nullptr;
+    LC_CUDA(cudaMalloc(&p, ctx->slot_bytes * 2));
+    ctx->d_staging = static_cast<uint8_t*>(p);
+    return LC_OK;
+}
+
+}  // namespace
+
+extern "C" lc_status lc_pack_device(lc_ctx* ctx, void* dst, uint64_t dst_capacity) {
+    g_err.clear();
+    if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_pack_device: ctx is NULL");
+    if (ctx->state != kSelected) return fail(LC_ERR_STATE, "lc_pack_device: call lc_select first");
+    const uint64_t bytes = ctx->hdr.bytes;
+    if (bytes > 0) {
+        if (!dst) return fail(LC_ERR_INVALID_ARG, "lc_pack_device: dst is NULL");
+        if (uintptr_t(dst) & 15) return fail(LC_ERR_INVALID_ARG, "lc_pack_device: dst must be 16-byte aligned");
+        if (bytes > dst_capacity)
+            return fail(LC_ERR_CAPACITY, "lc_pack_device: %llu bytes selected, capacity %llu",
+                        (unsigned long long)bytes, (unsigned long long)dst_capacity);
+        DeviceGuard g(ctx->device);
+        LC_TRY(check_device_ptr(dst, ctx->device, "lc_pack_device dst", true));
+        LC_TRY(launch_copy_range(ctx, ctx->d_pack_desc, ctx->hdr.n_pack_desc, kGather, 0, bytes,
+                                 static_cast<uint8_t*>(dst), ctx->stream));
+    }
+    ctx->state = kPacked;
+    return LC_OK;
+}
+
+extern "C" lc_status lc_pack_async(lc_ctx* ctx, lc_store* st) {
+    g_err.clear();
+    if (!ctx || !st) return fail(LC_ERR_INVALID_ARG, "lc_pack_async: NULL argument");
+    if (ctx->state != kSelected) return fail(LC_ERR_STATE, "lc_pack_async: call lc_select first");
+    if (st->nlayers != ctx->nlayers || st->layer_bytes != ctx->layer_bytes)
+        return fail(LC_ERR_INVALID_ARG, "lc_pack_async: store was created for another layout");
+    const uint64_t bytes = ctx->hdr.bytes;
+    DeviceGuard g(ctx->device);
+    if (bytes == 0) {
+        // nothing persisted: the step is durable as soon as earlier copies are
+        PendingPack pp;
+        pp.step = ctx->hdr.step;
+        pp.store = st;
+        LC_CUDA(cudaEventCreateWithFlags(&pp.done, cudaEventDisableTiming));
+        LC_CUDA(cudaEventRecord(pp.done, ctx->copy_stream));
+        ctx->pending.push_back(std::move(pp));
+        ctx->state = kPacked;
+        return LC_OK;
+    }
+    // reserve the destination of every selected layer block in the store
+    struct Extent { uint64_t soff; uint8_t* host; uint64_t len; };
+    std::vector<Extent> ext;
+    std::vector<StoreVersion> fresh;
+    if (st->per_layer == 0) {
+        if (st->top + bytes > st->capacity)
+            return fail(LC_ERR_CAPACITY, "lc_pack_async: store holds %llu of %llu bytes, %llu more needed",
+                        (unsigned long long)st->top, (unsigned long long)st->capacity,
+                        (unsigned long long)bytes);
+        ext.push_back({0, st->arena + st->top, bytes});
+        for (int32_t l = 0; l < ctx->nlayers; ++l) {
+            if (!ctx->mask[l]) continue;
+            fresh.push_back({st->next_id++, l, 0, ctx->hdr.step, st->top + ctx->offsets[l], ctx->layer_bytes[l], -1});
+        }
+        st->top += bytes;
+    } else {
+        for (int32_t l = 0; l < ctx->nlayers; ++l) {
+            if (!ctx->mask[l]) continue;
+            for (const StoreVersion& v : st->versions)
+                if (v.layer == l && !v.durable)
+                    return fail(LC_ERR_STATE,
+                                "lc_pack_async: layer %d still has a pending version (call lc_wait_durable)", l);
+        }
+        for (int32_t l = 0; l < ctx->nlayers; ++l) {
+            if (!ctx->mask[l]) continue;
+            const int32_t slot = int32_t(st->layer_writes[l] % st->per_layer);
+            const uint64_t off = st->layer_base[l] + uint64_t(slot) * st->layer_bytes[l];
+            st->versions.erase(std::remove_if(st->versions.begin(), st->versions.end(),
+                                              [&](const StoreVersion& v) { return v.layer == l && v.slot == slot; }),
+                               st->versions.end());
+            st->layer_writes[l] += 1;
+            ext.push_back({ctx->offsets[l], st->arena + off, ctx->layer_bytes[l]});
+            fresh.push_back({st->next_id++, l, 0, ctx->hdr.step, off, ctx->layer_bytes[l], slot});
+        }
+    }
+    LC_TRY(ensure_staging(ctx));
+    // forget copies into this store that have completed
+    st->inflight.erase(std::remove_if(st->inflight.begin(), st->inflight.end(),
+                                      [](cudaEvent_t ev) {
+                                          if (cudaEventQuery(ev) != cudaSuccess) return false;
+                                          cudaEventDestroy(ev);
+                                          return true;
+                                      }),
+                       st->inflight.end());
+    // ring: gather chunk c into slot c%2 on the stream, copy it out on the copy stream
+    const uint64_t S = ctx->slot_bytes;
+    for (uint64_t lo = 0, c = 0; lo < bytes; lo += S, ++c) {
+        const int r = int(c & 1);
+        const uint64_t hi = std::min(bytes, lo + S);
+        uint8_t* slot = ctx->d_staging + uint64_t(r) * S;
+        if (ctx->slot_busy[r]) LC_CUDA(cudaStreamWaitEvent(ctx->stream, ctx->ev_slot_free[r], 0));
+        LC_TRY(launch_copy_range(ctx, ctx->d_pack_desc, ctx->hdr.n_pack_desc, kGather, lo, hi, slot, ctx->stream));
+        LC_CUDA(cudaEventRecord(ctx->ev_slot_filled[r], ctx->stream));
+        LC_CUDA(cudaStreamWaitEvent(ctx->copy_stream, ctx->ev_slot_filled[r], 0));
+        for (const Extent& e : ext) {
+            const uint64_t a = std::max(lo, e.soff), b = std::min(hi, e.soff + e.len);
+            if (a >= b) continue;
+            LC_CUDA(cudaMemcpyAsync(e.host + (a - e.soff), slot + (a - lo), b - a, cudaMemcpyDeviceToHost,
+                                    ctx->copy_stream));
+            ctx->counters.d2h_bytes += b - a;
+        }
+        LC_CUDA(cudaEventRecord(ctx->ev_slot_free[r], ctx->copy_stream));
+        ctx->slot_busy[r] = true;
+    }
+    PendingPack pp;
+    pp.step = ctx->hdr.step;
+    pp.store = st;
+    LC_CUDA(cudaEventCreateWithFlags(&pp.done, cudaEventDisableTiming));
+    LC_CUDA(cudaEventRecord(pp.done, ctx->copy_stream));
+    cudaEvent_t inflight;
+    LC_CUDA(cudaEventCreateWithFlags(&inflight, cudaEventDisableTiming));
+    LC_CUDA(cudaEventRecord(inflight, ctx->copy_stream));
+    st->inflight.push_back(inflight);
+    for (const StoreVersion& v : fresh) {
+        st->versions.push_back(v);
+        pp.ids.push_back(v.id);
+    }
+    ctx->pending.push_back(std::move(pp));
+    ctx->state = kPacked;
+    return LC_OK;
+}
+
+extern "C" lc_status lc_commit_snapshot(lc_ctx* ctx) {
+    g_err.clear();
+    if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_commit_snapshot: ctx is NULL");
+    if (ctx->state == kSelected && ctx->hdr.n_selected == 0) {
+        ctx->state = kReady;
+        return LC_OK;
+    }
+    if (ctx->state != kPacked)
+        return fail(LC_ERR_STATE, "lc_commit_snapshot: the persisted layers were not packed");
+    if (ctx->cfg.mode == LC_DRIFT_SNAPSHOT && !ctx->cfg.fuse_commit && ctx->hdr.n_commit_desc > 0) {
+        DeviceGuard g(ctx->device);
+        LC_TRY(launch_copy_range(ctx, ctx->d_commit_desc, ctx->hdr.n_commit_desc, kCopy, 0,
+                                 ctx->hdr.commit_work, nullptr, ctx->stream));
+    }
+    ctx->state = kReady;
+    return LC_OK;
+}
+
+extern "C" lc_status lc_wait_durable(lc_ctx* ctx, int64_t step, int32_t timeout_ms) {
+    g_err.clear();
+    if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_wait_durable: ctx is NULL");
+    const int tmo = timeout_ms > 0 ? timeout_ms : ctx->cfg.timeout_ms;
+    DeviceGuard g(ctx->device);
+    bool found = false;
+    for (size_t i = 0; i < ctx->pending.size();) {
+        PendingPack& pp = ctx->pending[i];
+        if (pp.step != step) { ++i; continue; }
+        found = true;
+        LC_TRY(wait_event(pp.done, tmo, "lc_wait_durable"));
+        {
+            std::lock_guard<std::mutex> lk(g_store_mu);
+            if (g_live_stores.count(pp.store)) {
+                for (StoreVersion& v : pp.store->versions)
+                    if (std::find(pp.ids.begin(), pp.ids.end(), v.id) != pp.ids.end()) v.durable = 1;
+            }
+        }
+        cudaEventDestroy(pp.done);
+        ctx->pending.erase(ctx->pending.begin() + i);
+    }
+    if (!found) return fail(LC_ERR_NOT_FOUND, "lc_wait_durable: no pending pack of step %lld", (long long)step);
+    return LC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// restore (§3.5, Eq. 8)
+// ---------------------------------------------------------------------------
+extern "C" lc_status lc_restore(lc_ctx* ctx, lc_store* st, int64_t t_fail, int64_t* layer_steps_out) {
+    g_err.clear();
+    if (!ctx || !st) return fail(LC_ERR_INVALID_ARG, "lc_restore: NULL argument");
+    if (ctx->state == kNew) return fail(LC_ERR_STATE, "lc_restore: no layout registered");
+    if (step_open(ctx)) return fail(LC_ERR_STATE, "lc_restore: a step is open");
+    if (st->nlayers != ctx->nlayers || st->layer_bytes != ctx->layer_bytes)
+        return fail(LC_ERR_INVALID_ARG, "lc_restore: store was created for another layout");
+    const int32_t N = ctx->nlayers;
+    std::vector<int64_t> pick(N);
+    LC_TRY(lc_store_plan(st, t_fail, pick.data()));
+    DeviceGuard g(ctx->device);
+    LC_TRY(ensure_staging(ctx));
+
+    // restore stream: the picked blocks, layers ascending
+    std::vector<uint64_t> soff(N);
+    uint64_t total = 0;
+    for (int32_t l = 0; l < N; ++l) {
+        soff[l] = total;
+        total += ctx->layer_bytes[l];
+    }
+    const int32_t nsec = int32_t(ctx->secs.size());
+    std::vector<CopyDesc> desc(nsec);
+    for (int32_t l = 0; l < N; ++l) {
+        for (int32_t j = ctx->layer_sec_begin[l]; j < ctx->layer_sec_begin[l + 1]; ++j) {
+            const SectionDev& sec = ctx->secs[j];
+            const lc_segment& sg = ctx->segs[ctx->sec_seg[j]];
+            CopyDesc& d = desc[j];
+            d.woff = soff[l] + sec.off_in_layer;
+            d.nbytes = sec.nbytes;
+            d.span = sec.span;
+            d.src = nullptr;
+            const int part = ctx->sec_part[j];
+            d.dst = part == 0 ? static_cast<uint8_t*>(sg.w)
+                    : part == 1 ? reinterpret_cast<uint8_t*>(sg.exp_avg)
+                                : reinterpret_cast<uint8_t*>(sg.exp_avg_sq);
+            d.dst2 = part == 0 ? static_cast<uint8_t*>(sg.snap) : nullptr;
+        }
+    }
+    LC_CUDA(cudaMemcpyAsync(ctx->d_restore_desc, desc.data(), sizeof(CopyDesc) * nsec,
+                            cudaMemcpyHostToDevice, ctx->stream));
+    // the descriptor upload must land before the first scatter; the copy
+    // stream must not start overwriting staging before earlier users finish
+    cudaEvent_t ev_desc;
+    LC_CUDA(cudaEventCreateWithFlags(&ev_desc, cudaEventDisableTiming));
+    const uint64_t S = ctx->slot_bytes;
+    lc_status rc = LC_OK;
+    for (uint64_t lo = 0, c = 0; lo < total && rc == LC_OK; lo += S, ++c) {
+        const int r = int(c & 1);
+        const uint64_t hi = std::min(total, lo + S);
+        uint8_t* slot = ctx->d_staging + uint64_t(r) * S;
+        cudaError_t e = cudaSuccess;
+        if (ctx->slot_busy[r]) e = cudaStreamWaitEvent(ctx->copy_stream, ctx->ev_slot_free[r], 0);
+        for (int32_t l = 0; l < N && e == cudaSuccess; ++l) {
+            const uint64_t a = std::max(lo, soff[l]), b = std::min(hi, soff[l] + ctx->layer_bytes[l]);
+            if (a >= b) continue;
+            const StoreVersion& v = st->versions[size_t(pick[l])];
+            e = cudaMemcpyAsync(slot + (a - lo), st->arena + v.off + (a - soff[l]), b - a,
+                                cudaMemcpyHostToDevice, ctx->copy_stream);
+            ctx->counters.h2d_bytes += b - a;
+        }
+        if (e == cudaSuccess) e = cudaEventRecord(ctx->ev_slot_filled[r], ctx->copy_stream);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(ctx->stream, ctx->ev_slot_filled[r], 0);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            rc = fail(LC_ERR_CUDA, "lc_restore: %s", cudaGetErrorString(e));
+            break;
+        }
+        rc = launch_copy_range(ctx, ctx->d_restore_desc, nsec, kScatter, lo, hi, slot, ctx->stream);
+        if (rc == LC_OK && cudaEventRecord(ctx->ev_slot_free[r], ctx->stream) != cudaSuccess) {
+            cudaGetLastError();
+            rc = fail(LC_ERR_CUDA, "lc_restore: event record failed");
+        }
+        ctx->slot_busy[r] = true;
+    }
+    // per-layer state of the restored composite: t_l = version step, Delta_l = 0
+    std::vector<int64_t> steps(N);
+    for (int32_t l = 0; l < N; ++l) steps[l] = st->versions[size_t(pick[l])].step;
+    std::vector<double> zeros(N, 0.0);
+    if (rc == LC_OK) {
+        cudaError_t e = cudaMemcpyAsync(ctx->sp.t_last, steps.data(), sizeof(int64_t) * N,
+                                        cudaMemcpyHostToDevice, ctx->stream);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(ctx->sp.delta, zeros.data(), sizeof(double) * N, cudaMemcpyHostToDevice, ctx->stream);
+        if (e == cudaSuccess) e = cudaEventRecord(ev_desc, ctx->stream);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            rc = fail(LC_ERR_CUDA, "lc_restore: %s", cudaGetErrorString(e));
+        } else {
+            rc = wait_event(ev_desc, ctx->cfg.timeout_ms, "lc_restore");
+        }
+    }
+    cudaEventDestroy(ev_desc);
+    if (rc != LC_OK) return rc;
+    if (layer_steps_out) std::memcpy(layer_steps_out, steps.data(), sizeof(int64_t) * N);
+    ctx->last_step = t_fail;
+    ctx->state = kReady;
+    return LC_OK;
+}
+
+extern "C" lc_status lc_layer_block_bytes(const lc_ctx* ctx, int32_t layer, uint64_t* out) {
+    g_err.clear();
+    if (!ctx || !out) return fail(LC_ERR_INVALID_ARG, "lc_layer_block_bytes: NULL argument");
+    if (ctx->state == kNew) return fail(LC_ERR_STATE, "lc_layer_block_bytes: no layout registered");
+    if (layer < 0 || layer >= ctx->nlayers) return fail(LC_ERR_INVALID_ARG, "lc_layer_block_bytes: bad layer");
+    *out = ctx->layer_bytes[layer];
+    return LC_OK;
+}
+
+extern "C" lc_status lc_get_counters(const lc_ctx* ctx, lc_counters* out) {
+    g_err.clear();
+    if (!ctx || !out) return fail(LC_ERR_INVALID_ARG, "lc_get_counters: NULL argument");
+    *out = ctx->counters;
+    return LC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// stores
+// ---------------------------------------------------------------------------
+extern "C" lc_status lc_store_create(lc_store** out, const lc_ctx* ctx, uint64_t capacity_bytes,
+                                     int32_t versions_per_layer) {
+    g_err.clear();
+    if (!out || !ctx) return fail(LC_ERR_INVALID_ARG, "lc_store_create: NULL argument");
+    *out = nullptr;
+    if (ctx->state == kNew) return fail(LC_ERR_STATE, "lc_store_create: no layout registered");
+    if (versions_per_layer < 0 || versions_per_layer == 1)
+        return fail(LC_ERR_INVALID_ARG, "lc_store_create: versions_per_layer must be 0 or >= 2");
+    lc_store* st = new lc_store();
+    st->nlayers = ctx->nlayers;
+    st->per_layer = versions_per_layer;
+    st->layer_bytes = ctx->layer_bytes;
+    if (versions_per_layer == 0) {
+        if (capacity_bytes == 0) {
+            delete st;
+            return fail(LC_ERR_INVALID_ARG, "lc_store_create: capacity_bytes must be > 0");
+        }
+        st->capacity = capacity_bytes;
+    } else {
+        st->layer_base.resize(ctx->nlayers);
+        st->layer_writes.assign(ctx->nlayers, 0);
+        uint64_t off = 0;
+        for (int32_t l = 0; l < ctx->nlayers; ++l) {
+            st->layer_base[l] = off;
+            off += uint64_t(versions_per_layer) * ctx->layer_bytes[l];
+        }
+        st->capacity = off;
+    }
+    DeviceGuard g(ctx->device);
+    void* p = nullptr;
+    const cudaError_t e = cudaHostAlloc(&p, st->capacity, cudaHostAllocDefault);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        delete st;
+        return fail(LC_ERR_OOM, "lc_store_create: cannot pin %llu bytes: %s",
+                    (unsigned long long)st->capacity, cudaGetErrorString(e));
+    }
+    st->arena = static_cast<uint8_t*>(p);
+    {
+        std::lock_guard<std::mutex> lk(g_store_mu);
+        g_live_stores.insert(st);
+    }
+    *out = st;
+    return LC_OK;
+}
+
+namespace {
+
+// Waits (bounded) for copies still writing into a store's arena.
+lc_status drain_inflight(lc_store* st, int timeout_ms) {
+    lc_status rc = LC_OK;
+    for (cudaEvent_t ev : st->inflight) {
+        if (rc == LC_OK) rc = wait_event(ev, timeout_ms, "store copy");
+        cudaEventDestroy(ev);
+    }
+    st->inflight.clear();
+    return rc;
+}
+
+}  // namespace
+
+extern "C" void lc_store_destroy(lc_store* st) {
+    if (!st) return;
+    {
+        std::lock_guard<std::mutex> lk(g_store_mu);
+        g_live_stores.erase(st);
+    }
+    if (drain_inflight(st, 60000) == LC_OK && st->arena) cudaFreeHost(st->arena);
+    delete st;
+}
+
+extern "C" lc_status lc_store_clear(lc_store* st) {
+    g_err.clear();
+    if (!st) return fail(LC_ERR_INVALID_ARG, "lc_store_clear: store is NULL");
+    for (const StoreVersion& v : st->versions)
+        if (!v.durable) return fail(LC_ERR_STATE, "lc_store_clear: a version is still pending");
+    LC_TRY(drain_inflight(st, 60000));
+    st->versions.clear();
+    st->top = 0;
+    std::fill(st->layer_writes.begin(), st->layer_writes.end(), 0);
+    return LC_OK;
+}
+
+extern "C" int64_t lc_store_num_versions(const lc_store* st) {
+    return st ? int64_t(st->versions.size()) : 0;
+}
+
+extern "C" lc_status lc_store_get_version(const lc_store* st, int64_t index, lc_version* out) {
+    g_err.clear();
+    if (!st || !out) return fail(LC_ERR_INVALID_ARG, "lc_store_get_version: NULL argument");
+    if (index < 0 || index >= int64_t(st->versions.size()))
+        return fail(LC_ERR_INVALID_ARG, "lc_store_get_version: index %lld out of range", (long long)index);
+    const StoreVersion& v = st->versions[size_t(index)];
+    out->layer = v.layer;
+    out->durable = v.durable;
+    out->step = v.step;
+    out->host_ptr = st->arena + v.off;
+    out->bytes = v.bytes;
+    return LC_OK;
+}
+
+extern "C" lc_status lc_store_plan(const lc_store* st, int64_t t_fail, int64_t* pick_out) {
+    g_err.clear();
+    if (!st || !pick_out) return fail(LC_ERR_INVALID_ARG, "lc_store_plan: NULL argument");
+    for (int32_t l = 0; l < st->nlayers; ++l) pick_out[l] = -1;
+    for (size_t i = 0; i < st->versions.size(); ++i) {
+        const StoreVersion& v = st->versions[i];
+        if (!v.durable || v.step > t_fail) continue;
+        const int64_t cur = pick_out[v.layer];
+        if (cur < 0 || v.step >= st->versions[size_t(cur)].step) pick_out[v.layer] = int64_t(i);
+    }
+    for (int32_t l = 0; l < st->nlayers; ++l)
+        if (pick_out[l] < 0)
+            return fail(LC_ERR_NOT_FOUND, "lc_store_plan: layer %d has no durable version at or before step %lld",
+                        l, (long long)t_fail);
+    return LC_OK;
+}

@@ -1,0 +1,277 @@
+// lc_measure.cu -- Eq. 1 (§3.2) on sm_103a: per segment sum|W - R| and
+// sum|R|, combined per layer with the element count.
+//
+// Work decomposition: every segment is covered by 16-byte "virtual vectors"
+// aligned to absolute addresses (lc_internal.cuh).  All vectors of all
+// segments, layers ascending, form one linear work space that is cut into
+// G equal contiguous ranges, one per CTA, with G = resident CTAs on the
+// device (one wave).  A CTA streams its range with 128-bit non-allocating
+// loads of W and R, several in flight per thread, and writes one fp64
+// partial per (CTA, segment) run.  The last CTA to finish (atomic ticket, no
+// spinning) adds the partials of each segment, then the segments of each
+// layer, in a fixed order, so the result is deterministic for a layout.
+//
+// Precision: per-thread fp32 accumulators take at most kUnroll * kFlush
+// terms each before they are added (fixed tree) into per-thread fp64 sums;
+// the relative error of a layer sum is below about 2e-6 (all terms >= 0).
+#include "lc_internal.cuh"
+
+namespace lc {
+namespace {
+
+constexpr int kUnroll = 4;   // vectors of W (and of R) in flight per thread
+constexpr int kFlush = 4;    // unrolled iterations between fp64 flushes
+
+__device__ __forceinline__ uint4 ld_stream(const void* p) {
+    uint4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.L2::256B.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+    return v;
+}
+
+// Coherent load for R when the kernel also writes R (accumulate mode).
+__device__ __forceinline__ uint4 ld_coherent(const void* p) {
+    uint4 v;
+    asm volatile("ld.global.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p)
+                 : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void st_vec(void* p, uint4 v) {
+    asm volatile("st.global.v4.u32 [%0], {%1,%2,%3,%4};"
+                 :
+                 : "l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t x) { return __uint_as_float(x << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t x) { return __uint_as_float(x & 0xffff0000u); }
+
+// Adds one 16-byte vector pair into 8 fp32 lane accumulators.
+template <int ESZ_LOG2>
+__device__ __forceinline__ void accumulate(const uint4& w, const uint4& r, float (&ad)[8], float (&aa)[8]) {
+    const uint32_t wv[4] = {w.x, w.y, w.z, w.w};
+    const uint32_t rv[4] = {r.x, r.y, r.z, r.w};
+    if constexpr (ESZ_LOG2 == 1) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const float w0 = bf16_lo(wv[j]), w1 = bf16_hi(wv[j]);
+            const float r0 = bf16_lo(rv[j]), r1 = bf16_hi(rv[j]);
+            ad[2 * j] += fabsf(w0 - r0);
+            ad[2 * j + 1] += fabsf(w1 - r1);
+            aa[2 * j] += fabsf(r0);
+            aa[2 * j + 1] += fabsf(r1);
+        }
+    } else {
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const float w0 = __uint_as_float(wv[j]), r0 = __uint_as_float(rv[j]);
+            ad[j] += fabsf(w0 - r0);
+            aa[j] += fabsf(r0);
+        }
+    }
+}
+
+__device__ __forceinline__ float tree8(const float (&a)[8]) {
+    return ((a[0] + a[1]) + (a[2] + a[3])) + ((a[4] + a[5]) + (a[6] + a[7]));
+}
+
+// Full, co-aligned vectors [k0, k1) of one segment.
+template <int ESZ_LOG2, bool WRITE_R>
+__device__ __forceinline__ void run_vectors(const SegDev& sd, int64_t k0, int64_t k1,
+                                            double& dd, double& da) {
+    constexpr int BS = kMeasureThreads;
+    const uint8_t* wb = sd.w - (int64_t(sd.lead) << ESZ_LOG2);
+    uint8_t* rb = sd.r - (int64_t(sd.lead) << ESZ_LOG2);
+    int64_t k = k0 + threadIdx.x;
+    while (k < k1) {
+        float ad[8], aa[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) { ad[j] = 0.f; aa[j] = 0.f; }
+#pragma unroll 1
+        for (int f = 0; f < kFlush && k < k1; ++f) {
+            if (k + int64_t(kUnroll - 1) * BS < k1) {
+                uint4 w[kUnroll], r[kUnroll];
+#pragma unroll
+                for (int u = 0; u < kUnroll; ++u) {
+                    w[u] = ld_stream(wb + 16 * (k + int64_t(u) * BS));
+                    r[u] = WRITE_R ? ld_coherent(rb + 16 * (k + int64_t(u) * BS))
+                                   : ld_stream(rb + 16 * (k + int64_t(u) * BS));
+                }
+                if constexpr (WRITE_R) {
+#pragma unroll
+                    for (int u = 0; u < kUnroll; ++u) st_vec(rb + 16 * (k + int64_t(u) * BS), w[u]);
+                }
+#pragma unroll
+                for (int u = 0; u < kUnroll; ++u) accumulate<ESZ_LOG2>(w[u], r[u], ad, aa);
+                k += int64_t(kUnroll) * BS;
+            } else {
+                const uint4 w = ld_stream(wb + 16 * k);
+                const uint4 r = WRITE_R ? ld_coherent(rb + 16 * k) : ld_stream(rb + 16 * k);
+                if constexpr (WRITE_R) st_vec(rb + 16 * k, w);
+                accumulate<ESZ_LOG2>(w, r, ad, aa);
+                k += BS;
+            }
+        }
+        dd += double(tree8(ad));
+        da += double(tree8(aa));
+    }
+}
+
+__device__ __forceinline__ float load_elem(const uint8_t* base, int esz_log2, int64_t e) {
+    if (esz_log2 == 1) {
+        const uint16_t x = *reinterpret_cast<const uint16_t*>(base + 2 * e);
+        return __uint_as_float(uint32_t(x) << 16);
+    }
+    return *reinterpret_cast<const float*>(base + 4 * e);
+}
+
+// Vector k of a segment element by element (partial edge vectors, and every
+// vector of a segment whose W and R are not co-aligned).
+template <bool WRITE_R>
+__device__ void scalar_vector(const SegDev& sd, int64_t k, double& dd, double& da) {
+    const int ve = 16 >> sd.esz_log2;
+    for (int j = 0; j < ve; ++j) {
+        const int64_t e = k * ve - sd.lead + j;
+        if (e < 0 || e >= sd.numel) continue;
+        const float w = load_elem(sd.w, sd.esz_log2, e);
+        const float r = load_elem(sd.r, sd.esz_log2, e);
+        dd += double(fabsf(w - r));
+        da += double(fabsf(r));
+        if constexpr (WRITE_R) {
+            if (sd.esz_log2 == 1)
+                reinterpret_cast<uint16_t*>(sd.r)[e] = reinterpret_cast<const uint16_t*>(sd.w)[e];
+            else
+                reinterpret_cast<float*>(sd.r)[e] = reinterpret_cast<const float*>(sd.w)[e];
+        }
+    }
+}
+
+// Vectors [lo, hi) of one segment into the calling thread's fp64 sums.
+template <bool WRITE_R>
+__device__ void process_run(const SegDev& sd, int64_t lo, int64_t hi, double& dd, double& da) {
+    const int ve = 16 >> sd.esz_log2;
+    const bool head_partial = sd.lead > 0;
+    const bool tail_partial = ((int64_t(sd.lead) + sd.numel) % ve) != 0;
+    if (sd.coaligned) {
+        const int64_t kf0 = head_partial ? 1 : 0;
+        const int64_t kf1 = tail_partial ? sd.nvec - 1 : sd.nvec;
+        const int64_t a = lo > kf0 ? lo : kf0;
+        const int64_t b = hi < kf1 ? hi : kf1;
+        if (a < b) {
+            if (sd.esz_log2 == 1) run_vectors<1, WRITE_R>(sd, a, b, dd, da);
+            else run_vectors<2, WRITE_R>(sd, a, b, dd, da);
+        }
+        if (threadIdx.x == 0) {
+            if (head_partial && lo <= 0 && 0 < hi) scalar_vector<WRITE_R>(sd, 0, dd, da);
+            const int64_t last = sd.nvec - 1;
+            if (tail_partial && last >= lo && last < hi && !(head_partial && last == 0))
+                scalar_vector<WRITE_R>(sd, last, dd, da);
+        }
+    } else {
+        for (int64_t k = lo + threadIdx.x; k < hi; k += kMeasureThreads)
+            scalar_vector<WRITE_R>(sd, k, dd, da);
+    }
+}
+
+// Sum over the CTA in a fixed order; the result is valid in thread 0.
+__device__ __forceinline__ void block_sum(double& d, double& a, double* sd, double* sa) {
+    constexpr int kWarps = kMeasureThreads / 32;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        d += __shfl_down_sync(0xffffffffu, d, off);
+        a += __shfl_down_sync(0xffffffffu, a, off);
+    }
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (lane == 0) { sd[warp] = d; sa[warp] = a; }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double td = 0.0, ta = 0.0;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) { td += sd[w]; ta += sa[w]; }
+        d = td;
+        a = ta;
+    }
+    __syncthreads();
+}
+
+__device__ void finalize(const MeasureParams& p) {
+    for (int s = threadIdx.x; s < p.nseg; s += blockDim.x) {
+        double d = 0.0, a = 0.0;
+        for (int j = p.seg_slot_begin[s]; j < p.seg_slot_begin[s + 1]; ++j) {
+            const double2 v = __ldcg(&p.partials[j]);
+            d += v.x;
+            a += v.y;
+        }
+        p.seg_sums[2 * s] = d;
+        p.seg_sums[2 * s + 1] = a;
+    }
+    __syncthreads();
+    for (int l = threadIdx.x; l < p.nlayers; l += blockDim.x) {
+        double d = 0.0, a = 0.0;
+        int64_t n = 0;
+        for (int s = p.layer_seg_begin[l]; s < p.layer_seg_begin[l + 1]; ++s) {
+            d += __ldcg(&p.seg_sums[2 * s]);
+            a += __ldcg(&p.seg_sums[2 * s + 1]);
+            n += p.segs[s].numel;
+        }
+        p.sums[3 * l] = d;
+        p.sums[3 * l + 1] = a;
+        p.sums[3 * l + 2] = double(n);
+    }
+    if (threadIdx.x == 0) *p.ticket = 0u;
+}
+
+template <bool WRITE_R>
+__global__ void __launch_bounds__(kMeasureThreads) measure_kernel(const MeasureParams p) {
+    __shared__ double red_d[kMeasureThreads / 32];
+    __shared__ double red_a[kMeasureThreads / 32];
+    __shared__ unsigned int s_ticket;
+
+    const int b = blockIdx.x;
+    int64_t v0 = p.cta_vec_begin[b];
+    const int64_t v1 = p.cta_vec_begin[b + 1];
+    int s = p.cta_seg0[b];
+    int slot = p.cta_slot0[b];
+    while (v0 < v1 && s < p.nseg) {
+        const SegDev sd = p.segs[s];
+        const int64_t seg_end = sd.vec_begin + sd.nvec;
+        const int64_t lo = v0 - sd.vec_begin;
+        const int64_t hi = (v1 < seg_end ? v1 : seg_end) - sd.vec_begin;
+        double dd = 0.0, da = 0.0;
+        process_run<WRITE_R>(sd, lo, hi, dd, da);
+        block_sum(dd, da, red_d, red_a);
+        if (threadIdx.x == 0) p.partials[slot] = make_double2(dd, da);
+        ++slot;
+        ++s;
+        v0 = sd.vec_begin + hi;
+    }
+
+    if (threadIdx.x == 0) {
+        __threadfence();
+        s_ticket = atomicAdd(p.ticket, 1u);
+    }
+    __syncthreads();
+    if (s_ticket != gridDim.x - 1) return;
+    __threadfence();
+    finalize(p);
+}
+
+}  // namespace
+
+cudaError_t launch_measure(const MeasureParams& p, int grid, bool write_ref, cudaStream_t s) {
+    cudaGetLastError();  // a stale non-sticky status must not be blamed on this launch
+    if (write_ref) measure_kernel<true><<<grid, kMeasureThreads, 0, s>>>(p);
+    else measure_kernel<false><<<grid, kMeasureThreads, 0, s>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t measure_occupancy(int* blocks_per_sm) {
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, measure_kernel<false>,
+                                                         kMeasureThreads, 0);
+}
+
+}  // namespace lc
