@@ -285,6 +285,43 @@ lc_status lc_store_get_version(const lc_store* store, int64_t index, lc_version*
  * -1.  Returns NOT_FOUND if some layer has none. */
 lc_status lc_store_plan(const lc_store* store, int64_t t_fail, int64_t* pick_out);
 
+/* --- the measure without any device allocation -------------------------- */
+
+/* Limits of lc_measure_noalloc (its scratch is a fixed-size array). */
+#define LC_NOALLOC_MAX_SEGMENTS 512
+#define LC_NOALLOC_MAX_LAYERS 512
+#define LC_NOALLOC_SCRATCH_BYTES (192u * 1024u)
+
+/* The paper has no counterpart to this entry point; it exists for callers
+ * that cannot allocate device memory.  Some host programs must not call
+ * cudaMalloc once they are running: a framework that owns every byte of
+ * the GPU through its own memory pool, a process whose device footprint is
+ * fixed at start-up, or code where an allocation could synchronize the
+ * device at a bad moment.  Such a caller can still get the per-layer sums of
+ * Eq. 1 from this call without creating a context.
+ *
+ * Computes, on `cuda_stream` of `device`, the same per-layer sums as
+ * lc_measure: sums_out[3*l] = sum |W - R|, sums_out[3*l+1] = sum |R|,
+ * sums_out[3*l+2] = element count of layer l, for the segments `segs` (host
+ * array of nseg lc_segment, the layout rules of lc_register_layout; snap is
+ * only read, exp_avg / exp_avg_sq are ignored).  sums_out: caller-owned
+ * device memory of 3*nlayers fp64, 8-byte aligned.  Asynchronous; the host
+ * array may be reused when the call returns.
+ *
+ * Memory: the call allocates nothing.  Its scratch (tables, partial sums,
+ * completion counter) lives in one static device array of
+ * LC_NOALLOC_SCRATCH_BYTES that every GPU which loads the library holds
+ * until the process exits.  The first call on a device looks up that
+ * array's device address (cudaGetSymbolAddress) with the device current;
+ * make that first call before any stream capture.  All calls share the
+ * array: calls that overlap on the GPU (different streams, or different
+ * host threads, without ordering between them) race and give wrong sums.
+ *
+ * Errors: INVALID_ARG (layout, pointers), CAPACITY (nseg above
+ * LC_NOALLOC_MAX_SEGMENTS or nlayers above LC_NOALLOC_MAX_LAYERS), CUDA. */
+lc_status lc_measure_noalloc(int device, void* cuda_stream, const lc_segment* segs,
+                             int32_t nseg, int32_t nlayers, double* sums_out);
+
 #ifdef __cplusplus
 }
 #endif

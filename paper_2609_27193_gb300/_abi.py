@@ -83,7 +83,14 @@ SIGNATURES = {
     "lc_store_num_versions": (C.c_int64, [store_p]),
     "lc_store_get_version": (C.c_int, [store_p, C.c_int64, P(lc_version)]),
     "lc_store_plan": (C.c_int, [store_p, C.c_int64, C.c_void_p]),
+    "lc_measure_noalloc": (C.c_int, [C.c_int, C.c_void_p, P(lc_segment), C.c_int32, C.c_int32,
+                                     C.c_void_p]),
 }
+
+# limits of lc_measure_noalloc (include/layercheck.h)
+LC_NOALLOC_MAX_SEGMENTS = 512
+LC_NOALLOC_MAX_LAYERS = 512
+LC_NOALLOC_SCRATCH_BYTES = 192 * 1024
 
 _lib = None
 

@@ -212,6 +212,9 @@ extern "C" void lc_config_default(lc_config* cfg) {
 
 extern "C" const char* lc_last_error(void) { return g_err.c_str(); }
 
+// Lets other translation units of the library report an error message.
+void lc::set_last_error(const char* msg) { g_err = msg ? msg : ""; }
+
 extern "C" lc_status lc_create(lc_ctx** out, int device, void* cuda_stream, const lc_config* cfg) {
     g_err.clear();
     if (!out) return fail(LC_ERR_INVALID_ARG, "lc_create: out is NULL");

@@ -140,4 +140,7 @@ cudaError_t launch_select(const SelectParams& p, cudaStream_t s);
 cudaError_t launch_copy(const CopyParams& p, int grid, cudaStream_t s);
 cudaError_t copy_occupancy(int* blocks_per_sm);
 
+// Sets the thread-local message returned by lc_last_error().
+void set_last_error(const char* msg);
+
 }  // namespace lc
