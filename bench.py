@@ -51,6 +51,10 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--shape-blocks", type=int, default=0,
+                    help="keep only the first N transformer blocks (small case for kernel captures)")
+    ap.add_argument("--lean", action="store_true",
+                    help="no fp32 master weights in the generator (small case for kernel captures)")
     return ap.parse_args()
 
 
@@ -298,6 +302,18 @@ def reference_arm(args):
 # our arm
 # ---------------------------------------------------------------------------
 
+def first_blocks(shape, nblocks):
+    """The first `nblocks` transformer blocks of a shape, layers renumbered."""
+    from lc_workloads.shapes import ModelShape, TensorSpec
+    blocks = [l for l in range(shape.nlayers) if shape.layer_names[l].startswith("block")]
+    keep = blocks[:nblocks] if blocks else list(range(min(nblocks, shape.nlayers)))
+    ts = [TensorSpec(t.name, keep.index(t.layer), t.numel, t.dtype)
+          for t in shape.tensors if t.layer in keep]
+    sub = ModelShape("%s-first%d" % (shape.name, len(keep)), 0, 0, 0, 0, 0, 0, 0, False, False,
+                     ts, len(keep), [shape.layer_names[l] for l in keep])
+    return sub, keep
+
+
 def load_package():
     import paper_2609_27193_gb300 as P
     try:
@@ -324,11 +340,14 @@ def run_ours(args):
 
     wl = WORKLOADS[args.workload]
     shape = wl.shape()
+    base_scales = wl.layer_scales(shape)
+    if args.shape_blocks > 0:
+        shape, keep = first_blocks(shape, args.shape_blocks)
+        base_scales = base_scales[keep]
     tau = float(args.tau if args.tau is not None else wl.tau)
     K = wl.max_staleness
     t_setup = time.perf_counter()
-    st = gen.SyntheticState(shape, device=dev, seed=wl.seed + rank)
-    base_scales = wl.layer_scales(shape)
+    st = gen.SyntheticState(shape, device=dev, seed=wl.seed + rank, master=not args.lean)
     side = torch.cuda.Stream(device=dev)
     main = torch.cuda.current_stream(dev)
     lc = P.LayerCheck(device=local, stream=side)

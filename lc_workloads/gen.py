@@ -38,6 +38,8 @@ def _gen(device, *parts):
 class SyntheticState:
     """Device tensors of one workload.
 
+    master=False keeps no fp32 master copy (a smaller footprint for kernel
+    captures): the drift is then rounded into W at every step.
     alloc: "separate" -- one allocation per tensor (16-byte aligned);
            "flat"     -- one buffer per kind, tensors back to back, so a
                          tensor after an odd-sized one starts misaligned;
@@ -46,7 +48,7 @@ class SyntheticState:
     """
 
     def __init__(self, shape, device="cuda", seed=0, alloc="separate", moments=True,
-                 dtypes=None, moments_mask=None):
+                 dtypes=None, moments_mask=None, master=True):
         self.shape = shape
         self.device = torch.device(device)
         self.seed = int(seed)
@@ -56,6 +58,7 @@ class SyntheticState:
         self.dtypes = list(dtypes) if dtypes is not None else [t.dtype for t in self.specs]
         self.has_moments = ([bool(moments)] * nt if moments_mask is None else
                             [bool(moments) and bool(x) for x in moments_mask])
+        self.master = bool(master)
         self.W, self.R, self.M, self.m, self.v = [], [], [], [], []
         self._allocate()
         self.init()
@@ -82,7 +85,8 @@ class SyntheticState:
             for k, t in enumerate(self.specs):
                 self.W.append(torch.empty(t.numel, dtype=self._tdtype(k), device=dev))
                 self.R.append(torch.empty(t.numel, dtype=self._tdtype(k), device=dev))
-                self.M.append(torch.empty(t.numel, dtype=torch.float32, device=dev))
+                self.M.append(torch.empty(t.numel, dtype=torch.float32, device=dev)
+                              if self.master else None)
                 mo = self.has_moments[k]
                 self.m.append(torch.empty(t.numel, dtype=torch.float32, device=dev) if mo else None)
                 self.v.append(torch.empty(t.numel, dtype=torch.float32, device=dev) if mo else None)
@@ -114,7 +118,8 @@ class SyntheticState:
             b0 = offs[k]
             self.W.append(wbuf[b0:b0 + t.numel * esz].view(self._tdtype(k)))
             self.R.append(rbuf[b0 + sh:b0 + sh + t.numel * esz].view(self._tdtype(k)))
-            self.M.append(torch.empty(t.numel, dtype=torch.float32, device=dev))
+            self.M.append(torch.empty(t.numel, dtype=torch.float32, device=dev)
+                          if self.master else None)
             if self.has_moments[k]:
                 self.m.append(mbuf[fo:fo + t.numel])
                 self.v.append(vbuf[fo:fo + t.numel])
@@ -129,8 +134,11 @@ class SyntheticState:
         with torch.no_grad():
             for k in range(len(self.specs)):
                 g = _gen(self.device, self.seed, 0, k, 0)
-                self.M[k].normal_(0.0, 0.02, generator=g)
-                self.W[k].copy_(self.M[k])
+                if self.master:
+                    self.M[k].normal_(0.0, 0.02, generator=g)
+                    self.W[k].copy_(self.M[k])
+                else:
+                    self.W[k].normal_(0.0, 0.02, generator=g)
                 self.R[k].copy_(self.W[k])
                 self._draw_moments(0, k)
 
@@ -148,9 +156,12 @@ class SyntheticState:
                 if s > 0.0:
                     g = _gen(self.device, self.seed, step, k, 1)
                     noise = torch.randn(t.numel, generator=g, device=self.device, dtype=torch.float32)
-                    self.M[k].add_(noise, alpha=s * 0.02)
+                    if self.master:
+                        self.M[k].add_(noise, alpha=s * 0.02)
+                        self.W[k].copy_(self.M[k])
+                    else:      # lean mode: the drift is rounded into W every step
+                        self.W[k].add_(noise.mul_(s * 0.02).to(self.W[k].dtype))
                     del noise
-                    self.W[k].copy_(self.M[k])
                 if redraw_moments:
                     self._draw_moments(step, k)
 
@@ -158,8 +169,11 @@ class SyntheticState:
         """Overwrite W (and M) and/or R of tensor k with given float values."""
         with torch.no_grad():
             if w is not None:
-                self.M[k].copy_(torch.as_tensor(w, dtype=torch.float32))
-                self.W[k].copy_(self.M[k])
+                if self.master:
+                    self.M[k].copy_(torch.as_tensor(w, dtype=torch.float32))
+                    self.W[k].copy_(self.M[k])
+                else:
+                    self.W[k].copy_(torch.as_tensor(w, dtype=torch.float32))
             if r is not None:
                 self.R[k].copy_(torch.as_tensor(r, dtype=torch.float32))
 

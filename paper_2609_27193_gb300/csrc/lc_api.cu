@@ -389,19 +389,25 @@ extern "C" lc_status lc_register_layout(lc_ctx* ctx, const lc_segment* segs, int
     int occ = 0;
     LC_CUDA(measure_occupancy(&occ));
     if (occ <= 0) occ = 1;
-    const int64_t G = std::min<int64_t>(V, int64_t(ctx->sms) * occ);
+    const int64_t ngran_all = (V + LC_MEASURE_ALIGN_VECS - 1) / LC_MEASURE_ALIGN_VECS;
+    const int64_t G = std::min<int64_t>(ngran_all, int64_t(ctx->sms) * occ);
     ctx->measure_grid = int(G);
     std::vector<int64_t> cta_vec(G + 1);
     std::vector<int32_t> cta_seg0(G), cta_slot0(G);
     std::vector<int32_t> seg_slot_begin(nseg + 1, -1);
     int32_t slot = 0, s = 0;
-    for (int64_t b = 0; b <= G; ++b) cta_vec[b] = V * b / G;
+    {
+        // equal shares of the work space in granules of LC_MEASURE_ALIGN_VECS
+        const int64_t gran = LC_MEASURE_ALIGN_VECS;
+        const int64_t ngran = (V + gran - 1) / gran;
+        for (int64_t b = 0; b <= G; ++b) cta_vec[b] = std::min(V, ngran * b / G * gran);
+    }
     for (int64_t b = 0; b < G; ++b) {
         const int64_t v0 = cta_vec[b], v1 = cta_vec[b + 1];
         while (s < nseg && sd[s].vec_begin + sd[s].nvec <= v0) ++s;
         cta_seg0[b] = s;
         cta_slot0[b] = slot;
-        for (int32_t t = s; t < nseg && sd[t].vec_begin < v1; ++t) {
+        for (int32_t t = s; v0 < v1 && t < nseg && sd[t].vec_begin < v1; ++t) {
             if (seg_slot_begin[t] < 0) seg_slot_begin[t] = slot;
             ++slot;
         }

@@ -17,39 +17,59 @@ namespace {
 
 constexpr int BS = kCopyThreads;
 
+#ifndef LC_LD_PREFETCH
+#define LC_LD_PREFETCH 1
+#endif
+
 __device__ __forceinline__ uint4 ld_nc(const void* p) {
     uint4 v;
+#if LC_LD_PREFETCH
     asm volatile("ld.global.nc.L1::no_allocate.L2::256B.v4.u32 {%0,%1,%2,%3}, [%4];"
                  : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
                  : "l"(p));
+#else
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+#endif
     return v;
 }
 
+#ifndef LC_ST_CS
+#define LC_ST_CS 0
+#endif
+#ifndef LC_COPY_UNROLL
+#define LC_COPY_UNROLL 4
+#endif
+
 __device__ __forceinline__ void st_v4(void* p, uint4 v) {
+#if LC_ST_CS
+    asm volatile("st.global.cs.v4.u32 [%0], {%1,%2,%3,%4};"
+                 :
+                 : "l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                 : "memory");
+#else
     asm volatile("st.global.v4.u32 [%0], {%1,%2,%3,%4};"
                  :
                  : "l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
                  : "memory");
+#endif
 }
 
-// 16-byte vectors [v0, v1) of an entry.
+// 16-byte vectors [v0, v1) of an entry, LC_COPY_UNROLL loads in flight per thread.
 __device__ __forceinline__ void copy_vec(const uint8_t* src, uint8_t* dst, uint8_t* dst2,
                                          uint64_t v0, uint64_t v1) {
+    constexpr int U = LC_COPY_UNROLL;
     uint64_t v = v0 + threadIdx.x;
-    for (; v + 3 * BS < v1; v += 4 * BS) {
-        const uint4 x0 = ld_nc(src + 16 * v);
-        const uint4 x1 = ld_nc(src + 16 * (v + BS));
-        const uint4 x2 = ld_nc(src + 16 * (v + 2 * BS));
-        const uint4 x3 = ld_nc(src + 16 * (v + 3 * BS));
-        st_v4(dst + 16 * v, x0);
-        st_v4(dst + 16 * (v + BS), x1);
-        st_v4(dst + 16 * (v + 2 * BS), x2);
-        st_v4(dst + 16 * (v + 3 * BS), x3);
+    for (; v + (U - 1) * BS < v1; v += U * BS) {
+        uint4 x[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) x[u] = ld_nc(src + 16 * (v + uint64_t(u) * BS));
+#pragma unroll
+        for (int u = 0; u < U; ++u) st_v4(dst + 16 * (v + uint64_t(u) * BS), x[u]);
         if (dst2) {
-            st_v4(dst2 + 16 * v, x0);
-            st_v4(dst2 + 16 * (v + BS), x1);
-            st_v4(dst2 + 16 * (v + 2 * BS), x2);
-            st_v4(dst2 + 16 * (v + 3 * BS), x3);
+#pragma unroll
+            for (int u = 0; u < U; ++u) st_v4(dst2 + 16 * (v + uint64_t(u) * BS), x[u]);
         }
     }
     for (; v < v1; v += BS) {
@@ -117,9 +137,13 @@ __device__ void copy_entry(const CopyParams& p, const CopyDesc& d, uint64_t a, u
 }
 
 __global__ void __launch_bounds__(kCopyThreads) copy_kernel(const CopyParams p) {
+    // CTA ranges in granules of LC_COPY_ALIGN_BYTES (the last one ragged)
+    constexpr uint64_t kGran = LC_COPY_ALIGN_BYTES / 16;
     const uint64_t units = (p.hi - p.lo) >> 4;
-    const uint64_t u0 = units * blockIdx.x / gridDim.x;
-    const uint64_t u1 = units * (blockIdx.x + 1) / gridDim.x;
+    const uint64_t grans = (units + kGran - 1) / kGran;
+    uint64_t u0 = grans * blockIdx.x / gridDim.x * kGran;
+    uint64_t u1 = grans * (blockIdx.x + 1) / gridDim.x * kGran;
+    if (u1 > units) u1 = units;
     if (u0 >= u1 || p.ndesc <= 0) return;
     uint64_t x = p.lo + (u0 << 4);
     const uint64_t xe = p.lo + (u1 << 4);

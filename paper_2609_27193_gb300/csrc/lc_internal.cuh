@@ -11,6 +11,16 @@ constexpr int kMeasureThreads = 256;   // threads per measure CTA
 constexpr int kCopyThreads = 256;      // threads per copy CTA
 constexpr int kSelectThreads = 512;    // the select kernel is a single CTA
 
+// Work-range boundaries of the CTAs are rounded to these granules so that
+// every warp's 512-byte access starts on a 32-byte sector: a store that
+// covers only part of a sector makes L2 fetch the rest from DRAM first.
+#ifndef LC_MEASURE_ALIGN_VECS
+#define LC_MEASURE_ALIGN_VECS 32       // 16-byte vectors (512 bytes)
+#endif
+#ifndef LC_COPY_ALIGN_BYTES
+#define LC_COPY_ALIGN_BYTES 512
+#endif
+
 // One registered segment in measure order (layers ascending, registration
 // order within a layer).  The segment is covered by "virtual vectors":
 // 16-byte windows aligned to absolute 16-byte addresses of w; vector k

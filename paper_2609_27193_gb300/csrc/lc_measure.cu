@@ -19,14 +19,30 @@
 namespace lc {
 namespace {
 
-constexpr int kUnroll = 4;   // vectors of W (and of R) in flight per thread
-constexpr int kFlush = 4;    // unrolled iterations between fp64 flushes
+#ifndef LC_MEASURE_UNROLL
+#define LC_MEASURE_UNROLL 4
+#endif
+#ifndef LC_MEASURE_FLUSH
+#define LC_MEASURE_FLUSH 4
+#endif
+#ifndef LC_LD_PREFETCH
+#define LC_LD_PREFETCH 1
+#endif
+constexpr int kUnroll = LC_MEASURE_UNROLL;   // vectors of W (and of R) in flight per thread
+constexpr int kFlush = LC_MEASURE_FLUSH;     // unrolled iterations between fp64 flushes
+static_assert(kUnroll * kFlush <= 32, "fp32 partial sums are bounded to 32 terms");
 
 __device__ __forceinline__ uint4 ld_stream(const void* p) {
     uint4 v;
+#if LC_LD_PREFETCH
     asm volatile("ld.global.nc.L1::no_allocate.L2::256B.v4.u32 {%0,%1,%2,%3}, [%4];"
                  : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
                  : "l"(p));
+#else
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+#endif
     return v;
 }
 

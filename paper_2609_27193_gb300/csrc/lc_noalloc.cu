@@ -204,21 +204,26 @@ extern "C" lc_status lc_measure_noalloc(int device, void* cuda_stream, const lc_
         sd[i].vec_begin = V;
         V += sd[i].nvec;
     }
-    const int64_t G = V < ds.max_grid ? V : ds.max_grid;
+    const int64_t ngran_all = (V + LC_MEASURE_ALIGN_VECS - 1) / LC_MEASURE_ALIGN_VECS;
+    const int64_t G = ngran_all < ds.max_grid ? ngran_all : ds.max_grid;
     int64_t* cta_vec = reinterpret_cast<int64_t*>(t_image + kOffCtaVec);
     int32_t* cta_seg = reinterpret_cast<int32_t*>(t_image + kOffCtaSeg);
     int32_t* cta_slot = reinterpret_cast<int32_t*>(t_image + kOffCtaSlot);
     int32_t* seg_slot = reinterpret_cast<int32_t*>(t_image + kOffSegSlot);
     int32_t* layer_seg = reinterpret_cast<int32_t*>(t_image + kOffLayerSeg);
     for (int32_t i = 0; i <= nseg; ++i) seg_slot[i] = -1;
-    for (int64_t b = 0; b <= G; ++b) cta_vec[b] = V * b / G;
+    const int64_t ngran = (V + LC_MEASURE_ALIGN_VECS - 1) / LC_MEASURE_ALIGN_VECS;
+    for (int64_t b = 0; b <= G; ++b) {
+        const int64_t v = ngran * b / G * LC_MEASURE_ALIGN_VECS;
+        cta_vec[b] = v < V ? v : V;
+    }
     int32_t slot = 0, s = 0;
     for (int64_t b = 0; b < G; ++b) {
         const int64_t v0 = cta_vec[b], v1 = cta_vec[b + 1];
         while (s < nseg && sd[s].vec_begin + sd[s].nvec <= v0) ++s;
         cta_seg[b] = s;
         cta_slot[b] = slot;
-        for (int32_t t = s; t < nseg && sd[t].vec_begin < v1; ++t) {
+        for (int32_t t = s; v0 < v1 && t < nseg && sd[t].vec_begin < v1; ++t) {
             if (seg_slot[t] < 0) seg_slot[t] = slot;
             ++slot;
         }
