@@ -91,21 +91,27 @@ KERNEL_FILES = {"measure": ["lc_measure.cu", "lc_internal.cuh"],
                 "pack": ["lc_copy.cu", "lc_internal.cuh"]}
 
 
-def profiled_traffic(kernel, workload):
-    """dram bytes per launch from profiles/<kernel>_<workload>.md, if that
-    capture was taken of the current kernel source."""
+def profiled_traffic(kernel, workload, persisted_bytes=None):
+    """DRAM bytes per launch from profiles/<kernel>_<workload>.md, if that
+    capture was taken of the current kernel source: a fixed figure for the
+    measure, a per-persisted-byte figure scaled to the step for the pack."""
     path = os.path.join(ROOT, "profiles", "%s_%s.md" % (kernel, workload))
     try:
         text = open(path).read()
     except OSError:
         return None, None
     m_sha = re.search(r"source_sha256_16:\s*([0-9a-f]+)", text)
-    m_b = re.search(r"dram_bytes_per_full_launch:\s*([0-9.eE+]+)", text)
-    if not (m_sha and m_b):
+    m_full = re.search(r"dram_bytes_per_full_launch:\s*([0-9.eE+]+)", text)
+    m_per = re.search(r"dram_bytes_per_persisted_byte:\s*([0-9.eE+]+)", text)
+    if not m_sha or not (m_full or m_per):
         return None, None
     if m_sha.group(1) != kernel_source_sha(KERNEL_FILES[kernel]):
         return None, "stale"
-    return float(m_b.group(1)), os.path.relpath(path, ROOT)
+    if m_full:
+        return float(m_full.group(1)), os.path.relpath(path, ROOT)
+    if persisted_bytes is None:
+        return None, None
+    return float(m_per.group(1)) * persisted_bytes, os.path.relpath(path, ROOT)
 
 
 # ---------------------------------------------------------------------------
@@ -314,6 +320,22 @@ def first_blocks(shape, nblocks):
     return sub, keep
 
 
+def d2h_link_probe(torch, dev, nbytes=4 << 30):
+    """Plain device->pinned-host copy bandwidth measured beside the e2e loop
+    (the host link is shared with other jobs on the machine, so it varies)."""
+    d = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    h = torch.empty(nbytes, dtype=torch.uint8, pin_memory=True)
+    best = 0.0
+    for _ in range(3):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        h.copy_(d, non_blocking=True)
+        torch.cuda.synchronize()
+        best = max(best, nbytes / (time.perf_counter() - t0) / 1e9)
+    del d, h
+    return best
+
+
 def load_package():
     import paper_2609_27193_gb300 as P
     try:
@@ -456,9 +478,11 @@ def run_ours(args):
     pack_gbs = (statistics.mean(pbytes) / (statistics.mean(pack_ms) / 1e3) / 1e9
                 if statistics.mean(pack_ms) > 0 else 0.0)
     dominant = "measure" if sum(measure_ms) >= sum(pack_ms) else "pack"
-    traffic, tsrc = profiled_traffic(dominant, args.workload)
-    if traffic is not None and dominant == "pack":
-        traffic = None      # pack traffic depends on the step's selection
+    mean_persisted = statistics.mean(r["nbytes"] for r in recs)
+    traffic, tsrc = profiled_traffic(dominant, args.workload,
+                                     mean_persisted if dominant == "pack" else None)
+    if args.shape_blocks or args.lean:
+        traffic, tsrc = None, None       # the profiles describe the full layout
     achieved = meas_gbs if dominant == "measure" else pack_gbs
     roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
                 "frac": achieved / hbm, "traffic": traffic, "kernel": dominant,
@@ -485,6 +509,7 @@ def run_ours(args):
             pass
         cap = full if avail == 0 else min(full, int(avail * 0.6))
         store = P.Store(lc, capacity_bytes=cap)
+        link = d2h_link_probe(torch, dev)
         e_recs, e_bytes = [], []
         for i in range(max(1, args.warmup) + args.steps):
             t += 1
@@ -499,6 +524,7 @@ def run_ours(args):
                "d2h_bytes_per_step": int(d2h),
                "ms_per_step": 1e3 * e_s / len(e_recs),
                "d2h_GBps": d2h / (statistics.mean(r["host_s"] - r["decision_s"] for r in e_recs)) / 1e9,
+               "d2h_link_GBps_measured": link,
                "note": "weights, snapshot and moments are device-resident training state; the "
                        "step's only host traffic is the decision block and the persisted "
                        "layers copied into the pinned store"}

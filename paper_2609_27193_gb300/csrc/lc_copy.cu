@@ -36,10 +36,10 @@ __device__ __forceinline__ uint4 ld_nc(const void* p) {
 }
 
 #ifndef LC_ST_CS
-#define LC_ST_CS 0
+#define LC_ST_CS 1
 #endif
 #ifndef LC_COPY_UNROLL
-#define LC_COPY_UNROLL 4
+#define LC_COPY_UNROLL 8
 #endif
 
 __device__ __forceinline__ void st_v4(void* p, uint4 v) {
