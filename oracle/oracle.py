@@ -26,33 +26,36 @@ class _Tensor(C.Structure):
 def lib():
     global _lib
     if _lib is None:
-        path = build_oracle()
-        L = C.CDLL(path)
-        L.lco_bf16_value.restype = C.c_double
-        L.lco_bf16_value.argtypes = [C.c_uint16]
-        L.lco_layer_sums.restype = None
-        L.lco_layer_sums.argtypes = [C.POINTER(_Tensor), C.c_int32, C.POINTER(C.c_double)]
-        L.lco_update_measure.restype = C.c_double
-        L.lco_update_measure.argtypes = [C.c_double] * 4
-        L.lco_select_step.restype = C.c_int32
-        L.lco_select_step.argtypes = [C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
-                                      C.c_void_p, C.c_double, C.c_int32, C.c_int64,
-                                      C.c_int32, C.c_void_p, C.POINTER(C.c_int32)]
-        L.lco_staleness.restype = None
-        L.lco_staleness.argtypes = [C.c_int32, C.c_void_p, C.c_void_p, C.c_int64,
-                                    C.POINTER(C.c_int64), C.POINTER(C.c_double)]
-        L.lco_layer_block_bytes.restype = C.c_uint64
-        L.lco_layer_block_bytes.argtypes = [C.POINTER(_Tensor), C.c_int32, C.c_uint32]
-        L.lco_pack_layer.restype = C.c_uint64
-        L.lco_pack_layer.argtypes = [C.POINTER(_Tensor), C.c_int32, C.c_uint32, C.c_void_p]
-        L.lco_unpack_layer.restype = C.c_int32
-        L.lco_unpack_layer.argtypes = [C.c_void_p, C.c_uint64, C.POINTER(_Tensor),
-                                       C.c_int32, C.c_uint32]
-        L.lco_composite_pick.restype = None
-        L.lco_composite_pick.argtypes = [C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
-                                         C.c_int32, C.c_int64, C.c_void_p]
-        _lib = L
+        _lib = declare(C.CDLL(build_oracle()))
     return _lib
+
+
+def declare(L):
+    """Sets the ctypes signatures of an oracle library and returns it."""
+    L.lco_bf16_value.restype = C.c_double
+    L.lco_bf16_value.argtypes = [C.c_uint16]
+    L.lco_layer_sums.restype = None
+    L.lco_layer_sums.argtypes = [C.POINTER(_Tensor), C.c_int32, C.POINTER(C.c_double)]
+    L.lco_update_measure.restype = C.c_double
+    L.lco_update_measure.argtypes = [C.c_double] * 4
+    L.lco_select_step.restype = C.c_int32
+    L.lco_select_step.argtypes = [C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
+                                  C.c_void_p, C.c_double, C.c_int32, C.c_int64,
+                                  C.c_int32, C.c_void_p, C.POINTER(C.c_int32)]
+    L.lco_staleness.restype = None
+    L.lco_staleness.argtypes = [C.c_int32, C.c_void_p, C.c_void_p, C.c_int64,
+                                C.POINTER(C.c_int64), C.POINTER(C.c_double)]
+    L.lco_layer_block_bytes.restype = C.c_uint64
+    L.lco_layer_block_bytes.argtypes = [C.POINTER(_Tensor), C.c_int32, C.c_uint32]
+    L.lco_pack_layer.restype = C.c_uint64
+    L.lco_pack_layer.argtypes = [C.POINTER(_Tensor), C.c_int32, C.c_uint32, C.c_void_p]
+    L.lco_unpack_layer.restype = C.c_int32
+    L.lco_unpack_layer.argtypes = [C.c_void_p, C.c_uint64, C.POINTER(_Tensor),
+                                   C.c_int32, C.c_uint32]
+    L.lco_composite_pick.restype = None
+    L.lco_composite_pick.argtypes = [C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
+                                     C.c_int32, C.c_int64, C.c_void_p]
+    return L
 
 
 class Tensor:

@@ -170,10 +170,11 @@ def test_power_of_two_scaling_is_invariant(oracle_lib):
 def test_sums_depend_on_reference_not_current_for_denominator(oracle_lib):
     # The denominator is mean |W(t-1)|: swapping W and R changes A but not D.
     w = bf16_bits([1.0, 3.0])
-    r = bf16_bits([2.0, 2.0])
+    r = bf16_bits([2.0, 4.0])
     d1, a1, _ = O.layer_sums([O.Tensor(w, r)])
     d2, a2, _ = O.layer_sums([O.Tensor(r, w)])
-    assert d1 == d2 == 2.0 and a1 == 4.0 and a2 == 4.0
+    assert d1 == d2 == 2.0 and a1 == 6.0 and a2 == 4.0
+    r = bf16_bits([2.0, 2.0])
     w2 = bf16_bits([-1.0, -3.0])
     d3, a3, _ = O.layer_sums([O.Tensor(w2, r)])
     assert d3 == 8.0 and a3 == 4.0        # |(-1)-2| + |(-3)-2|, not |w|-|r|
@@ -302,8 +303,13 @@ def test_table1_default_layer_writes(oracle_lib):
 
 
 def test_staleness_closed_form(oracle_lib):
-    mx, wt = O.staleness([0, 5, 10], [1, 1, 2], 10)
-    assert mx == 10 and wt == (1 * 10 + 1 * 5 + 2 * 0) / 4
+    # §3.3: larger layers count proportionally more in the weighted average
+    mx, wt = O.staleness([0, 5, 10], [3, 1, 2], 10)
+    assert mx == 10 and wt == (3 * 10 + 1 * 5 + 2 * 0) / 6
+    mx, wt = O.staleness([7, 7], [1000, 1], 9)
+    assert mx == 2 and wt == 2.0
+    mx, wt = O.staleness([4, 0], [1, 1000], 4)
+    assert mx == 4 and wt == 4000 / 1001
 
 
 def test_select_rejects_bad_arguments(oracle_lib):
