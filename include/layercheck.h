@@ -79,7 +79,9 @@ typedef enum { LC_DRIFT_SNAPSHOT = 0, LC_DRIFT_ACCUMULATE = 1 } lc_drift_mode;
  *   w          : device, numel elements, current weights W_l(t); must be
  *                aligned to its element size (written only by lc_restore)
  *   snap       : device, numel elements of w_dtype, the reference weights R
- *                (written by commit / accumulate mode / restore)
+ *                (written by commit / accumulate mode / restore); may be
+ *                NULL in LC_DRIFT_ACCUMULATE mode for a context that measures
+ *                only through lc_adamw_step_measure (lc_measure then fails)
  *   exp_avg    : device, numel fp32 Adam first moment, or NULL
  *   exp_avg_sq : device, numel fp32 Adam second moment; NULL iff exp_avg is
  *   numel      : > 0
@@ -257,6 +259,46 @@ lc_status lc_layer_block_bytes(const lc_ctx* ctx, int32_t layer, uint64_t* out);
 
 /* Library-side work counters of the context. */
 lc_status lc_get_counters(const lc_ctx* ctx, lc_counters* out);
+
+/* --- fused optimizer step with the drift read off the update ------------ */
+
+/* Optimizer inputs of one segment, in the registration order of
+ * lc_register_layout.  The segment's w must be its fp32 (master) weights and
+ * its exp_avg / exp_avg_sq must be set.
+ *   grad       : device, numel elements of grad_dtype (LC_BF16 or LC_F32)
+ *   model_copy : device, numel bf16 elements that receive the updated
+ *                weights rounded to nearest even (e.g. the model's bf16
+ *                parameters), or NULL */
+typedef struct {
+    const void* grad;
+    int32_t grad_dtype;
+    int32_t reserved;
+    void* model_copy;
+} lc_optim_segment;
+
+/* AdamW hyperparameters (decoupled weight decay). */
+typedef struct {
+    double lr, beta1, beta2, eps, weight_decay;
+} lc_adamw_hparams;
+
+/* Registers the gradient and model-copy pointers of every segment (§3.4.2:
+ * the drift is computed on the optimizer update path).  Requires a layout
+ * in LC_DRIFT_ACCUMULATE mode whose segments all have fp32 w and Adam
+ * moments.  Errors: STATE (no layout, or snapshot mode), INVALID_ARG. */
+lc_status lc_register_optimizer(lc_ctx* ctx, const lc_optim_segment* segs, int32_t nseg);
+
+/* One AdamW step on every registered segment, in place on w, exp_avg and
+ * exp_avg_sq (and model_copy), with the Eq. 1 sums of the update taken on
+ * the same pass: D_l = sum |w_new - w_old|, A_l = sum |w_old|, so W(t-1) is
+ * the weights before this update and no separate scan reads them again.
+ * Takes the place of lc_measure for the step (then lc_select accumulates,
+ * Eq. 2).  step = t >= 1 is also the bias-correction count.  fp32
+ * arithmetic, one rounding per operation in this order: p *= 1 - lr*wd;
+ * m = beta1*m + (1-beta1)*g; v = beta2*v + (1-beta2)*(g*g);
+ * p -= lr * ((m / (1-beta1^t)) / (sqrt(v / (1-beta2^t)) + eps)); the fp32
+ * constants are formed in binary64 and rounded once.  Asynchronous.
+ * Errors: STATE (no optimizer registered, or a step is open), INVALID_ARG. */
+lc_status lc_adamw_step_measure(lc_ctx* ctx, int64_t step, const lc_adamw_hparams* hp);
 
 /* --- persisted-version store (pinned host memory) ---------------------- */
 

@@ -225,3 +225,86 @@ void lco_composite_pick(int32_t nversions, const int32_t* v_layer,
             pick_out[l] = i;
     }
 }
+
+/* ------------------------------------------------------------------------
+ * AdamW with the drift read off the update (§3.4.2).
+ *
+ * AdamW (Adam with decoupled weight decay) per element, with step count t:
+ *   p  <- p * (1 - lr*wd)                       decoupled weight decay
+ *   m  <- beta1*m + (1-beta1)*g                 first moment
+ *   v  <- beta2*v + (1-beta2)*g*g               second moment
+ *   p  <- p - lr * (m/(1-beta1^t)) / (sqrt(v/(1-beta2^t)) + eps)
+ * in binary32, the precision of the optimizer state, one rounding per
+ * operation in exactly this order.
+ * ---------------------------------------------------------------------- */
+void lco_adamw_constants(const lco_adamw* hp, int64_t t, float out[9])
+{
+    out[0] = (float)(1.0 - hp->lr * hp->weight_decay);
+    out[1] = (float)hp->beta1;
+    out[2] = (float)(1.0 - hp->beta1);
+    out[3] = (float)hp->beta2;
+    out[4] = (float)(1.0 - hp->beta2);
+    out[5] = (float)(1.0 - pow(hp->beta1, (double)t));
+    out[6] = (float)(1.0 - pow(hp->beta2, (double)t));
+    out[7] = (float)hp->lr;
+    out[8] = (float)hp->eps;
+}
+
+uint16_t lco_bf16_round(float f)
+{
+    uint32_t u;
+    memcpy(&u, &f, sizeof u);
+    if ((u & 0x7f800000u) == 0x7f800000u && (u & 0x007fffffu))
+        return (uint16_t)((u >> 16) | 0x0040u);          /* quiet NaN */
+    /* nearest, ties to the even bf16: add half an ulp minus one, plus the
+     * parity of the bit that stays */
+    uint32_t keep_lsb = (u >> 16) & 1u;
+    return (uint16_t)((u + 0x7fffu + keep_lsb) >> 16);
+}
+
+void lco_adamw_step(const lco_adamw* hp, int64_t t, int64_t n, float* p, float* m, float* v,
+                    const void* grad, int32_t grad_bf16, uint16_t* model,
+                    double* d_out, double* a_out)
+{
+    float c[9];
+    lco_adamw_constants(hp, t, c);
+    const float decay = c[0], b1 = c[1], omb1 = c[2], b2 = c[3], omb2 = c[4];
+    const float bc1 = c[5], bc2 = c[6], lr = c[7], eps = c[8];
+    double d_sum = 0.0, a_sum = 0.0;
+    for (int64_t i = 0; i < n; ++i) {
+        float g;
+        if (grad_bf16) {
+            uint16_t bits;
+            memcpy(&bits, (const uint8_t*)grad + 2 * i, sizeof bits);
+            g = (float)lco_bf16_value(bits);
+        } else {
+            memcpy(&g, (const uint8_t*)grad + 4 * i, sizeof g);
+        }
+        const float p_old = p[i];
+        const float p_decayed = p_old * decay;
+        const float m1a = b1 * m[i];
+        const float m1b = omb1 * g;
+        const float m_new = m1a + m1b;
+        const float gg = g * g;
+        const float v1a = b2 * v[i];
+        const float v1b = omb2 * gg;
+        const float v_new = v1a + v1b;
+        const float m_hat = m_new / bc1;
+        const float v_hat = v_new / bc2;
+        const float root = sqrtf(v_hat);
+        const float denom = root + eps;
+        const float step_dir = m_hat / denom;
+        const float step = lr * step_dir;
+        const float p_new = p_decayed - step;
+        p[i] = p_new;
+        m[i] = m_new;
+        v[i] = v_new;
+        if (model)
+            model[i] = lco_bf16_round(p_new);
+        /* Eq. 1 terms: W(t) - W(t-1) and W(t-1), exact in binary64 */
+        d_sum += fabs((double)p_new - (double)p_old);
+        a_sum += fabs((double)p_old);
+    }
+    *d_out = d_sum;
+    *a_out = a_sum;
+}

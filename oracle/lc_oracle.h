@@ -9,9 +9,11 @@
  * baseline of the benchmark may load it; the product library never does,
  * and the two share no source, header, table or helper.
  *
- * All floating-point arithmetic is IEEE binary64, summed in the plain
- * order the definitions state (tensor registration order, then element
- * index order).  Build with -ffp-contract=off so no multiply-add is fused.
+ * Floating-point arithmetic is IEEE binary64, summed in the plain order the
+ * definitions state (tensor registration order, then element index order),
+ * except the AdamW step, which runs in binary32, the precision of the
+ * optimizer state it updates.  Build with -ffp-contract=off so no
+ * multiply-add is fused.
  */
 #ifndef LC_ORACLE_H
 #define LC_ORACLE_H
@@ -85,6 +87,32 @@ int32_t lco_unpack_layer(const uint8_t* src, uint64_t nbytes, lco_tensor* t,
 void lco_composite_pick(int32_t nversions, const int32_t* v_layer,
                         const int64_t* v_step, const uint8_t* v_durable,
                         int32_t nlayers, int64_t t_fail, int64_t* pick_out);
+
+/* AdamW hyperparameters of one optimizer step (binary64, as given by the
+ * training script). */
+typedef struct {
+    double lr, beta1, beta2, eps, weight_decay;
+} lco_adamw;
+
+/* fp32 constants of one AdamW step at step count t >= 1: out[0] = 1 - lr*wd,
+ * out[1] = beta1, out[2] = 1 - beta1, out[3] = beta2, out[4] = 1 - beta2,
+ * out[5] = 1 - beta1^t, out[6] = 1 - beta2^t, out[7] = lr, out[8] = eps;
+ * each formed in binary64 and rounded once to binary32. */
+void lco_adamw_constants(const lco_adamw* hp, int64_t t, float out[9]);
+
+/* One AdamW step (decoupled weight decay) on n fp32 parameters in place,
+ * with the drift sums of Eq. 1 taken on the same pass (§3.4.2: the drift is
+ * read off the optimizer update): d_out = sum |p_new - p_old|, a_out =
+ * sum |p_old| (binary64 sums of the binary32 values).  grad is bf16 bits
+ * (grad_bf16 = 1) or fp32.  model (nullable) receives bf16(p_new) rounded
+ * to nearest even.  Every fp32 operation rounds once, in the order written
+ * in lc_oracle.c. */
+void lco_adamw_step(const lco_adamw* hp, int64_t t, int64_t n, float* p, float* m, float* v,
+                    const void* grad, int32_t grad_bf16, uint16_t* model,
+                    double* d_out, double* a_out);
+
+/* Round-to-nearest-even binary32 -> bf16 bits (NaN -> quiet NaN). */
+uint16_t lco_bf16_round(float f);
 
 #ifdef __cplusplus
 }

@@ -17,6 +17,11 @@ SNAPSHOT, ACCUMULATE = 0, 1
 _lib = None
 
 
+class AdamW(C.Structure):
+    _fields_ = [("lr", C.c_double), ("beta1", C.c_double), ("beta2", C.c_double),
+                ("eps", C.c_double), ("weight_decay", C.c_double)]
+
+
 class _Tensor(C.Structure):
     _fields_ = [("w", C.c_void_p), ("r", C.c_void_p), ("m", C.c_void_p),
                 ("v", C.c_void_p), ("numel", C.c_int64), ("dtype", C.c_int32),
@@ -52,6 +57,14 @@ def declare(L):
     L.lco_unpack_layer.restype = C.c_int32
     L.lco_unpack_layer.argtypes = [C.c_void_p, C.c_uint64, C.POINTER(_Tensor),
                                    C.c_int32, C.c_uint32]
+    L.lco_adamw_constants.restype = None
+    L.lco_adamw_constants.argtypes = [C.POINTER(AdamW), C.c_int64, C.POINTER(C.c_float)]
+    L.lco_bf16_round.restype = C.c_uint16
+    L.lco_bf16_round.argtypes = [C.c_float]
+    L.lco_adamw_step.restype = None
+    L.lco_adamw_step.argtypes = [C.POINTER(AdamW), C.c_int64, C.c_int64, C.c_void_p, C.c_void_p,
+                                 C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p,
+                                 C.POINTER(C.c_double), C.POINTER(C.c_double)]
     L.lco_composite_pick.restype = None
     L.lco_composite_pick.argtypes = [C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
                                      C.c_int32, C.c_int64, C.c_void_p]
@@ -161,3 +174,30 @@ def composite_pick(v_layer, v_step, v_durable, nlayers, t_fail):
     lib().lco_composite_pick(v_layer.size, _ptr(v_layer), _ptr(v_step), _ptr(v_durable),
                              nlayers, int(t_fail), _ptr(pick))
     return pick
+
+
+def adamw_constants(hp, t):
+    out = (C.c_float * 9)()
+    lib().lco_adamw_constants(C.byref(AdamW(*hp)), int(t), out)
+    return list(out)
+
+
+def bf16_round(f):
+    return int(lib().lco_bf16_round(float(f)))
+
+
+def adamw_step(hp, t, p, m, v, grad, model=None):
+    """One AdamW step in place on float32 arrays p, m, v; grad is uint16
+    (bf16 bits) or float32; model (uint16, nullable) receives bf16(p).
+    Returns (D, A) of Eq. 1 for the update.  hp = (lr, beta1, beta2, eps, wd)."""
+    for a in (p, m, v):
+        assert a.dtype == np.float32 and a.flags.c_contiguous
+    grad = np.ascontiguousarray(grad)
+    is_bf16 = grad.dtype == np.uint16
+    assert is_bf16 or grad.dtype == np.float32
+    if model is not None:
+        assert model.dtype == np.uint16 and model.flags.c_contiguous
+    d, a = C.c_double(0), C.c_double(0)
+    lib().lco_adamw_step(C.byref(AdamW(*hp)), int(t), p.size, _ptr(p), _ptr(m), _ptr(v),
+                         _ptr(grad), int(is_bf16), _ptr(model), C.byref(d), C.byref(a))
+    return d.value, a.value

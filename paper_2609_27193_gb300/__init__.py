@@ -37,13 +37,15 @@ def _dtype_code(t):
 
 
 def segment(layer, w, snap, exp_avg=None, exp_avg_sq=None):
-    """An lc_segment over torch CUDA tensors (contiguous, same numel)."""
+    """An lc_segment over torch CUDA tensors (contiguous, same numel); snap
+    may be None in accumulate mode (fused optimizer path only)."""
     for name, t in (("w", w), ("snap", snap), ("exp_avg", exp_avg), ("exp_avg_sq", exp_avg_sq)):
         if t is not None and not t.is_contiguous():
             raise ValueError("%s must be contiguous" % name)
-    if snap.dtype != w.dtype or snap.numel() != w.numel():
+    if snap is not None and (snap.dtype != w.dtype or snap.numel() != w.numel()):
         raise ValueError("snap must match w in dtype and size")
-    return lc_segment(int(layer), _dtype_code(w), w.data_ptr(), snap.data_ptr(),
+    return lc_segment(int(layer), _dtype_code(w), w.data_ptr(),
+                      snap.data_ptr() if snap is not None else None,
                       exp_avg.data_ptr() if exp_avg is not None else None,
                       exp_avg_sq.data_ptr() if exp_avg_sq is not None else None,
                       int(w.numel()))
@@ -107,6 +109,26 @@ class LayerCheck:
 
     def measure(self, step):
         check(self._lib.lc_measure(self._ctx, int(step)))
+
+    def register_optimizer(self, grads, model_copies=None):
+        """Gradients (and optional bf16 model copies) of every segment, in the
+        order of register_layout, for the fused AdamW + drift step."""
+        from ._abi import lc_optim_segment
+        n = len(grads)
+        arr = (lc_optim_segment * n)()
+        for i, g in enumerate(grads):
+            mc = None if model_copies is None else model_copies[i]
+            arr[i] = lc_optim_segment(g.data_ptr(), _dtype_code(g), 0,
+                                      mc.data_ptr() if mc is not None else None)
+        self._keep.append((grads, model_copies))
+        check(self._lib.lc_register_optimizer(self._ctx, arr, n))
+
+    def adamw_step_measure(self, step, lr, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.0):
+        """One fused AdamW step on every segment with the Eq. 1 sums of the
+        update (takes the place of measure)."""
+        from ._abi import lc_adamw_hparams
+        hp = lc_adamw_hparams(float(lr), float(beta1), float(beta2), float(eps), float(weight_decay))
+        check(self._lib.lc_adamw_step_measure(self._ctx, int(step), C.byref(hp)))
 
     def layer_sums_ptr(self):
         p = C.c_void_p()

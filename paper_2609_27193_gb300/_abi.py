@@ -47,6 +47,16 @@ class lc_version(C.Structure):
                 ("host_ptr", C.c_void_p), ("bytes", C.c_uint64)]
 
 
+class lc_optim_segment(C.Structure):
+    _fields_ = [("grad", C.c_void_p), ("grad_dtype", C.c_int32), ("reserved", C.c_int32),
+                ("model_copy", C.c_void_p)]
+
+
+class lc_adamw_hparams(C.Structure):
+    _fields_ = [("lr", C.c_double), ("beta1", C.c_double), ("beta2", C.c_double),
+                ("eps", C.c_double), ("weight_decay", C.c_double)]
+
+
 class lc_counters(C.Structure):
     _fields_ = [("kernel_launches", C.c_int64), ("measure_launches", C.c_int64),
                 ("select_launches", C.c_int64), ("copy_launches", C.c_int64),
@@ -83,6 +93,8 @@ SIGNATURES = {
     "lc_store_num_versions": (C.c_int64, [store_p]),
     "lc_store_get_version": (C.c_int, [store_p, C.c_int64, P(lc_version)]),
     "lc_store_plan": (C.c_int, [store_p, C.c_int64, C.c_void_p]),
+    "lc_register_optimizer": (C.c_int, [ctx_p, P(lc_optim_segment), C.c_int32]),
+    "lc_adamw_step_measure": (C.c_int, [ctx_p, C.c_int64, P(lc_adamw_hparams)]),
     "lc_measure_noalloc": (C.c_int, [C.c_int, C.c_void_p, P(lc_segment), C.c_int32, C.c_int32,
                                      C.c_void_p]),
 }

@@ -167,6 +167,9 @@ struct lc_ctx {
     std::vector<int32_t> sec_part;         // 0 = W, 1 = exp_avg, 2 = exp_avg_sq
     int measure_grid = 0, copy_grid = 0, nslots = 0;
     bool any_write_ref = false;
+    std::vector<int32_t> order;            // measure position -> registration index
+    bool snap_missing = false;             // some segment has no snapshot
+    OptSegDev* d_opt = nullptr;            // optimizer table (lc_register_optimizer)
 
     // device memory
     void* d_tables = nullptr;
@@ -276,6 +279,7 @@ extern "C" void lc_destroy(lc_ctx* ctx) {
     }
     for (auto& pp : ctx->pending) cudaEventDestroy(pp.done);
     cudaFree(ctx->d_tables);
+    cudaFree(ctx->d_opt);
     cudaFree(ctx->d_staging);
     if (ctx->h_result) cudaFreeHost(ctx->h_result);
     if (ctx->ev_result) cudaEventDestroy(ctx->ev_result);
@@ -322,19 +326,25 @@ extern "C" lc_status lc_register_layout(lc_ctx* ctx, const lc_segment* segs, int
         if (s.w_dtype != LC_BF16 && s.w_dtype != LC_F32)
             return fail(LC_ERR_INVALID_ARG, "segment %d: unknown dtype %d", i, s.w_dtype);
         if (s.numel <= 0) return fail(LC_ERR_INVALID_ARG, "segment %d: numel must be > 0", i);
-        if (!s.w || !s.snap) return fail(LC_ERR_INVALID_ARG, "segment %d: w and snap are required", i);
+        if (!s.w) return fail(LC_ERR_INVALID_ARG, "segment %d: w is required", i);
+        if (!s.snap && ctx->cfg.mode != LC_DRIFT_ACCUMULATE)
+            return fail(LC_ERR_INVALID_ARG, "segment %d: snap is required in snapshot mode", i);
         if ((s.exp_avg == nullptr) != (s.exp_avg_sq == nullptr))
             return fail(LC_ERR_INVALID_ARG, "segment %d: exp_avg and exp_avg_sq must both be set or both NULL", i);
         const uintptr_t esz = s.w_dtype == LC_BF16 ? 2 : 4;
         if ((uintptr_t(s.w) % esz) || (uintptr_t(s.snap) % esz))
             return fail(LC_ERR_INVALID_ARG, "segment %d: w/snap not aligned to the element size", i);
+        if (s.snap && s.snap == s.w)
+            return fail(LC_ERR_INVALID_ARG, "segment %d: snap must not alias w", i);
         if (s.exp_avg && ((uintptr_t(s.exp_avg) % 4) || (uintptr_t(s.exp_avg_sq) % 4)))
             return fail(LC_ERR_INVALID_ARG, "segment %d: Adam moments not 4-byte aligned", i);
         char what[64];
         snprintf(what, sizeof what, "segment %d w", i);
         LC_TRY(check_device_ptr(s.w, ctx->device, what, false));
-        snprintf(what, sizeof what, "segment %d snap", i);
-        LC_TRY(check_device_ptr(s.snap, ctx->device, what, false));
+        if (s.snap) {
+            snprintf(what, sizeof what, "segment %d snap", i);
+            LC_TRY(check_device_ptr(s.snap, ctx->device, what, false));
+        }
         if (s.exp_avg) {
             snprintf(what, sizeof what, "segment %d exp_avg", i);
             LC_TRY(check_device_ptr(s.exp_avg, ctx->device, what, false));
@@ -363,6 +373,9 @@ extern "C" lc_status lc_register_layout(lc_ctx* ctx, const lc_segment* segs, int
     ctx->nlayers = nlayers;
     ctx->segs.resize(nseg);
     for (int32_t i = 0; i < nseg; ++i) ctx->segs[i] = segs[order[i]];
+    ctx->order = order;
+    ctx->snap_missing = false;
+    for (int32_t i = 0; i < nseg; ++i) ctx->snap_missing |= segs[i].snap == nullptr;
     ctx->layer_seg_begin.assign(nlayers + 1, 0);
     for (int32_t i = 0; i < nseg; ++i) ctx->layer_seg_begin[ctx->segs[i].layer + 1] += 1;
     for (int32_t l = 0; l < nlayers; ++l) ctx->layer_seg_begin[l + 1] += ctx->layer_seg_begin[l];
@@ -380,7 +393,7 @@ extern "C" lc_status lc_register_layout(lc_ctx* ctx, const lc_segment* segs, int
         d.numel = s.numel;
         d.lead = int32_t((uintptr_t(s.w) & 15) >> esz_log2);
         d.esz_log2 = esz_log2;
-        d.coaligned = (uintptr_t(s.w) & 15) == (uintptr_t(s.snap) & 15);
+        d.coaligned = s.snap && (uintptr_t(s.w) & 15) == (uintptr_t(s.snap) & 15);
         d.layer = s.layer;
         d.nvec = (int64_t(d.lead) + s.numel + ve - 1) / ve;
         d.vec_begin = V;
@@ -577,8 +590,98 @@ extern "C" lc_status lc_measure(lc_ctx* ctx, int64_t step) {
     if (step < 0 || step <= ctx->last_step)
         return fail(LC_ERR_INVALID_ARG, "lc_measure: step %lld must exceed the previous step %lld",
                     (long long)step, (long long)ctx->last_step);
+    if (ctx->snap_missing)
+        return fail(LC_ERR_STATE, "lc_measure: a segment has no snapshot (use lc_adamw_step_measure)");
     DeviceGuard g(ctx->device);
     LC_CUDA(launch_measure(ctx->mp, ctx->measure_grid, ctx->cfg.mode == LC_DRIFT_ACCUMULATE, ctx->stream));
+    ctx->counters.kernel_launches += 1;
+    ctx->counters.measure_launches += 1;
+    ctx->last_step = step;
+    ctx->state = kMeasured;
+    return LC_OK;
+}
+
+extern "C" lc_status lc_register_optimizer(lc_ctx* ctx, const lc_optim_segment* osegs, int32_t nseg) {
+    g_err.clear();
+    if (!ctx || !osegs) return fail(LC_ERR_INVALID_ARG, "lc_register_optimizer: NULL argument");
+    if (ctx->state == kNew) return fail(LC_ERR_STATE, "lc_register_optimizer: no layout registered");
+    if (ctx->cfg.mode != LC_DRIFT_ACCUMULATE)
+        return fail(LC_ERR_STATE, "lc_register_optimizer: the fused step needs LC_DRIFT_ACCUMULATE mode");
+    if (nseg != ctx->nseg)
+        return fail(LC_ERR_INVALID_ARG, "lc_register_optimizer: %d segments, the layout has %d", nseg, ctx->nseg);
+    DeviceGuard g(ctx->device);
+    std::vector<OptSegDev> od(ctx->nseg);
+    for (int32_t pos = 0; pos < ctx->nseg; ++pos) {
+        const int32_t i = ctx->order[pos];
+        const lc_segment& s = ctx->segs[pos];
+        const lc_optim_segment& o = osegs[i];
+        if (s.w_dtype != LC_F32)
+            return fail(LC_ERR_INVALID_ARG, "segment %d: the fused step updates fp32 weights", i);
+        if (!s.exp_avg) return fail(LC_ERR_INVALID_ARG, "segment %d: the fused step needs Adam moments", i);
+        if (!o.grad || (o.grad_dtype != LC_BF16 && o.grad_dtype != LC_F32))
+            return fail(LC_ERR_INVALID_ARG, "segment %d: gradient pointer or dtype invalid", i);
+        const uintptr_t gesz = o.grad_dtype == LC_BF16 ? 2 : 4;
+        if (uintptr_t(o.grad) % gesz || uintptr_t(o.model_copy) % 2)
+            return fail(LC_ERR_INVALID_ARG, "segment %d: gradient or model copy misaligned", i);
+        char what[64];
+        snprintf(what, sizeof what, "segment %d grad", i);
+        LC_TRY(check_device_ptr(o.grad, ctx->device, what, false));
+        if (o.model_copy) {
+            snprintf(what, sizeof what, "segment %d model_copy", i);
+            LC_TRY(check_device_ptr(o.model_copy, ctx->device, what, false));
+        }
+        OptSegDev& d = od[pos];
+        d.grad = static_cast<const uint8_t*>(o.grad);
+        d.model = static_cast<uint8_t*>(o.model_copy);
+        d.m = s.exp_avg;
+        d.v = s.exp_avg_sq;
+        d.grad_bf16 = o.grad_dtype == LC_BF16;
+        // vectors of w start at w - 4*lead (16-byte aligned); every other array
+        // must line up with them for the vector path
+        const uintptr_t w0 = uintptr_t(s.w) & ~uintptr_t(15);
+        const uintptr_t lead = (uintptr_t(s.w) & 15) / 4;
+        bool fast = (uintptr_t(s.exp_avg) - 4 * lead) % 16 == 0 && (uintptr_t(s.exp_avg_sq) - 4 * lead) % 16 == 0;
+        fast = fast && (d.grad_bf16 ? (uintptr_t(o.grad) - 2 * lead) % 8 == 0
+                                    : (uintptr_t(o.grad) - 4 * lead) % 16 == 0);
+        if (o.model_copy) fast = fast && (uintptr_t(o.model_copy) - 2 * lead) % 8 == 0;
+        (void)w0;
+        d.fast = fast ? 1 : 0;
+    }
+    if (!ctx->d_opt) {
+        void* p = nullptr;
+        LC_CUDA(cudaMalloc(&p, sizeof(OptSegDev) * ctx->nseg));
+        ctx->d_opt = static_cast<OptSegDev*>(p);
+    }
+    LC_CUDA(cudaMemcpy(ctx->d_opt, od.data(), sizeof(OptSegDev) * ctx->nseg, cudaMemcpyHostToDevice));
+    return LC_OK;
+}
+
+extern "C" lc_status lc_adamw_step_measure(lc_ctx* ctx, int64_t step, const lc_adamw_hparams* hp) {
+    g_err.clear();
+    if (!ctx || !hp) return fail(LC_ERR_INVALID_ARG, "lc_adamw_step_measure: NULL argument");
+    if (!ctx->d_opt) return fail(LC_ERR_STATE, "lc_adamw_step_measure: no optimizer registered");
+    if (step_open(ctx)) return fail(LC_ERR_STATE, "lc_adamw_step_measure: the previous step is still open");
+    if (step < 1 || step <= ctx->last_step)
+        return fail(LC_ERR_INVALID_ARG, "lc_adamw_step_measure: step %lld must be >= 1 and exceed %lld",
+                    (long long)step, (long long)ctx->last_step);
+    const double vals[5] = {hp->lr, hp->beta1, hp->beta2, hp->eps, hp->weight_decay};
+    for (double x : vals)
+        if (!std::isfinite(x)) return fail(LC_ERR_INVALID_ARG, "lc_adamw_step_measure: non-finite hyperparameter");
+    if (!(hp->beta1 >= 0.0 && hp->beta1 < 1.0 && hp->beta2 >= 0.0 && hp->beta2 < 1.0) || hp->lr < 0.0 ||
+        hp->eps < 0.0)
+        return fail(LC_ERR_INVALID_ARG, "lc_adamw_step_measure: hyperparameters out of range");
+    AdamConsts c;
+    c.decay = float(1.0 - hp->lr * hp->weight_decay);
+    c.b1 = float(hp->beta1);
+    c.omb1 = float(1.0 - hp->beta1);
+    c.b2 = float(hp->beta2);
+    c.omb2 = float(1.0 - hp->beta2);
+    c.bc1 = float(1.0 - std::pow(hp->beta1, double(step)));
+    c.bc2 = float(1.0 - std::pow(hp->beta2, double(step)));
+    c.lr = float(hp->lr);
+    c.eps = float(hp->eps);
+    DeviceGuard g(ctx->device);
+    LC_CUDA(launch_adamw_measure(ctx->mp, ctx->d_opt, c, ctx->measure_grid, ctx->stream));
     ctx->counters.kernel_launches += 1;
     ctx->counters.measure_launches += 1;
     ctx->last_step = step;

@@ -143,9 +143,30 @@ struct SelectParams {
     int32_t fuse_commit;
 };
 
+// Optimizer inputs of one segment in measure order (fused AdamW step).
+struct OptSegDev {
+    const uint8_t* grad;   // bf16 or fp32 gradient
+    uint8_t* model;        // bf16 model copy, or null
+    float* m;              // exp_avg
+    float* v;              // exp_avg_sq
+    int32_t grad_bf16;
+    int32_t fast;          // W, m, v, grad and model line up with W's 16-byte vectors
+};
+
+// fp32 constants of one AdamW step (formed in binary64, rounded once).
+struct AdamConsts {
+    float decay;           // 1 - lr*wd
+    float b1, omb1;        // beta1, 1 - beta1
+    float b2, omb2;        // beta2, 1 - beta2
+    float bc1, bc2;        // 1 - beta1^t, 1 - beta2^t
+    float lr, eps;
+};
+
 // Launchers (return the launch error, if any).
 cudaError_t launch_measure(const MeasureParams& p, int grid, bool write_ref, cudaStream_t s);
 cudaError_t measure_occupancy(int* blocks_per_sm);
+cudaError_t launch_adamw_measure(const MeasureParams& p, const OptSegDev* opt, const AdamConsts& c,
+                                 int grid, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, cudaStream_t s);
 cudaError_t launch_copy(const CopyParams& p, int grid, cudaStream_t s);
 cudaError_t copy_occupancy(int* blocks_per_sm);

@@ -54,6 +54,18 @@ MUTATIONS = [
      ["test_composite_pick_equals_replay", "test_crash_before_durable_uses_previous_version"]),
     ("composite-first-not-latest", "v_step[i] >= v_step[pick_out[l]]", "0",
      ["test_composite_pick_equals_replay", "test_composite_equals_latest_persisted_versions"]),
+    ("adamw-no-bias-correction", "const float m_hat = m_new / bc1;", "const float m_hat = m_new;",
+     ["test_adamw_hand_cases", "test_constant_gradient_closed_form"]),
+    ("adamw-second-moment-linear", "const float gg = g * g;", "const float gg = g;",
+     ["test_adamw_hand_cases", "test_matches_binary64_adamw_within_fp32_rounding"]),
+    ("adamw-decay-dropped", "const float p_decayed = p_old * decay;", "const float p_decayed = p_old;",
+     ["test_adamw_hand_cases"]),
+    ("adamw-drift-against-decayed", "d_sum += fabs((double)p_new - (double)p_old);",
+     "d_sum += fabs((double)p_new - (double)p_decayed);",
+     ["test_adamw_hand_cases", "test_fused_drift_sums_are_eq1_of_the_update"]),
+    ("bf16-round-truncates", "return (uint16_t)((u + 0x7fffu + keep_lsb) >> 16);",
+     "return (uint16_t)(u >> 16); (void)keep_lsb;", ["test_fused_drift_sums_are_eq1_of_the_update",
+                                                      "test_bf16_round_matches_torch"]),
 ]
 
 RUNNER = r"""
@@ -61,14 +73,14 @@ import ctypes, sys
 sys.path.insert(0, sys.argv[1])
 from oracle import oracle as O
 O._lib = O.declare(ctypes.CDLL(sys.argv[2]))
-from tests import test_oracle_pins as pins
+from tests import test_oracle_pins as pins, test_oracle_adamw as pins_adamw
 failed = []
 for name in sys.argv[3:]:
-    fn = pins.__dict__[name]
+    fn = pins.__dict__.get(name) or pins_adamw.__dict__[name]
     args = fn.__code__.co_varnames[:fn.__code__.co_argcount]
-    kw = {k: v for k, v in (("align", 256), ("dtype", "bf16")) if k in args}
+    kw = {k: v for k, v in (("oracle_lib", None), ("align", 256), ("dtype", "bf16")) if k in args}
     try:
-        fn(None, **kw)
+        fn(**kw)
     except Exception as e:
         failed.append(name)
 print("FAILED:" + ",".join(failed))
