@@ -53,6 +53,9 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--shape-blocks", type=int, default=0,
                     help="keep only the first N transformer blocks (small case for kernel captures)")
+    ap.add_argument("--path", choices=["scan", "fused"], default="scan",
+                    help="scan: measure against the snapshot (default); fused: AdamW step with "
+                         "the drift read off the update, fp32 master weights")
     ap.add_argument("--lean", action="store_true",
                     help="no fp32 master weights in the generator (small case for kernel captures)")
     return ap.parse_args()
@@ -87,7 +90,8 @@ def kernel_source_sha(files):
     return h.hexdigest()[:16]
 
 
-KERNEL_FILES = {"measure": ["lc_measure.cu", "lc_internal.cuh"],
+KERNEL_FILES = {"measure": ["lc_measure.cu", "lc_reduce.cuh", "lc_internal.cuh"],
+                "fused_adamw": ["lc_adamw.cu", "lc_reduce.cuh", "lc_internal.cuh"],
                 "pack": ["lc_copy.cu", "lc_internal.cuh"]}
 
 
@@ -170,6 +174,16 @@ class ClockSampler:
 # algorithmic bytes
 # ---------------------------------------------------------------------------
 
+# lr, beta1, beta2, eps, weight decay of the fused path (lr as in the paper's runs)
+FUSED_HP = (1e-5, 0.9, 0.999, 1e-8, 0.01)
+
+
+def fused_step_bytes(state):
+    """AdamW step per param: read w, m, v (fp32) and the bf16 gradient, write
+    w, m, v and the bf16 model copy: 28 B; the drift sums add no traffic."""
+    return sum(28 * t.numel for t in state.specs)
+
+
 def measure_bytes(state, accumulate=False):
     tot = 0
     for k, t in enumerate(state.specs):
@@ -178,12 +192,12 @@ def measure_bytes(state, accumulate=False):
     return tot
 
 
-def layer_payload_bytes(state):
+def layer_payload_bytes(state, fp32_weights=False):
     """Per layer: W bytes + moment bytes (the payload of its packed block)."""
     out = [0] * state.nlayers
     wb = [0] * state.nlayers
     for k, t in enumerate(state.specs):
-        esz = 2 if state.dtypes[k] == "bf16" else 4
+        esz = 4 if fp32_weights or state.dtypes[k] != "bf16" else 2
         out[t.layer] += t.numel * esz + (8 * t.numel if state.has_moments[k] else 0)
         wb[t.layer] += t.numel * esz
     return out, wb
@@ -369,20 +383,34 @@ def run_ours(args):
     tau = float(args.tau if args.tau is not None else wl.tau)
     K = wl.max_staleness
     t_setup = time.perf_counter()
-    st = gen.SyntheticState(shape, device=dev, seed=wl.seed + rank, master=not args.lean)
+    fused = args.path == "fused"
+    st = gen.SyntheticState(shape, device=dev, seed=wl.seed + rank,
+                            master=fused or not args.lean, snapshot=not fused)
     side = torch.cuda.Stream(device=dev)
     main = torch.cuda.current_stream(dev)
-    lc = P.LayerCheck(device=local, stream=side)
-    lc.register_layout([P.segment(t.layer, st.W[k], st.R[k], st.m[k], st.v[k])
-                        for k, t in enumerate(shape.tensors)], shape.nlayers)
+    grads = grad_bias = None
+    if fused:
+        # fp32 master weights are the optimizer's parameters; the bf16 W is the
+        # model copy the step refreshes; no snapshot is kept
+        lc = P.LayerCheck(device=local, stream=side, mode=P.LC_DRIFT_ACCUMULATE)
+        lc.register_layout([P.segment(t.layer, st.M[k], None, st.m[k], st.v[k])
+                            for k, t in enumerate(shape.tensors)], shape.nlayers)
+        grads = [torch.empty(t.numel, dtype=torch.bfloat16, device=dev) for t in shape.tensors]
+        lc.register_optimizer(grads, st.W)
+        # per-layer gradient bias: layers with consistent gradients move faster
+        grad_bias = gen.u_shape(shape.nlayers, 2.0, 0.05, 0.3, np.random.default_rng(wl.seed + 7))
+    else:
+        lc = P.LayerCheck(device=local, stream=side)
+        lc.register_layout([P.segment(t.layer, st.W[k], st.R[k], st.m[k], st.v[k])
+                            for k, t in enumerate(shape.tensors)], shape.nlayers)
     sums = None
     if world > 1:
         sums = torch.zeros(3 * shape.nlayers, dtype=torch.float64, device=dev)
         lc.set_layer_sums_buffer(sums)
     full = sum(lc.layer_block_bytes(l) for l in range(shape.nlayers))
     dst = torch.empty(full, dtype=torch.uint8, device=dev)
-    payload, wbytes = layer_payload_bytes(st)
-    mbytes = measure_bytes(st)
+    payload, wbytes = layer_payload_bytes(st, fp32_weights=fused)
+    mbytes = fused_step_bytes(st) if fused else measure_bytes(st)
     gemm = None
     if args.workload == "8b-cadence":
         a = torch.randn(8192, 8192, device=dev, dtype=torch.bfloat16)
@@ -403,8 +431,19 @@ def run_ours(args):
         # inputs would stay L2-resident between steps: overwrite L2 before each one
         flush = torch.empty(4 * l2_bytes, dtype=torch.uint8, device=dev)
 
+    def new_inputs(t):
+        if not fused:
+            st.drift(t, scales_for(t))
+            return
+        g = torch.Generator(device=dev)
+        for k, spec in enumerate(shape.tensors):
+            g.manual_seed(gen.mix_seed(wl.seed, t, k, 5))
+            tmp = torch.randn(spec.numel, generator=g, device=dev)
+            grads[k].copy_(tmp.add_(float(grad_bias[spec.layer])).mul_(1e-3))
+            del tmp
+
     def step(t, mode, store=None):
-        st.drift(t, scales_for(t))
+        new_inputs(t)
         if flush is not None:
             flush.fill_(t & 0xFF)
         side.wait_stream(main)
@@ -418,7 +457,10 @@ def run_ours(args):
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
         h0 = time.perf_counter()
         ev[0].record(side)
-        lc.measure(t)
+        if fused:
+            lc.adamw_step_measure(t, FUSED_HP[0], FUSED_HP[1], FUSED_HP[2], FUSED_HP[3], FUSED_HP[4])
+        else:
+            lc.measure(t)
         ev[1].record(side)
         if sums is not None:
             import torch.distributed as dist
@@ -469,7 +511,7 @@ def run_ours(args):
     select_ms = [ms(r, 1, 2) for r in recs]
     pack_ms = [ms(r, 2, 3) for r in recs]
     decision_ms = [1e3 * r["decision_s"] for r in recs]
-    pbytes = [pack_bytes(r["mask"], payload, wbytes) for r in recs]
+    pbytes = [pack_bytes(r["mask"], payload, wbytes, fused_commit=not fused) for r in recs]
     tot_bytes = sum(mbytes + pb for pb in pbytes)
     tot_s = sum(step_ms) / 1e3
     frac_sel = float(np.mean([r["mask"].mean() for r in recs]))
@@ -486,19 +528,23 @@ def run_ours(args):
     pack_gbs = (statistics.mean(pbytes) / (statistics.mean(pack_ms) / 1e3) / 1e9
                 if statistics.mean(pack_ms) > 0 else 0.0)
     dominant = "measure" if sum(measure_ms) >= sum(pack_ms) else "pack"
+    measure_name = "fused_adamw" if fused else "measure"
     mean_persisted = statistics.mean(r["nbytes"] for r in recs)
-    traffic, tsrc = profiled_traffic(dominant, args.workload,
-                                     mean_persisted if dominant == "pack" else None)
+    traffic, tsrc = profiled_traffic(measure_name if dominant == "measure" else "pack",
+                                     args.workload, mean_persisted if dominant == "pack" else None)
+    if fused and dominant == "pack":
+        traffic, tsrc = None, None       # the pack profile is of bf16 weights
     if args.shape_blocks or args.lean:
         traffic, tsrc = None, None       # the profiles describe the full layout
     achieved = meas_gbs if dominant == "measure" else pack_gbs
     roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                "frac": achieved / hbm, "traffic": traffic, "kernel": dominant,
+                "frac": achieved / hbm, "traffic": traffic,
+                "kernel": measure_name if dominant == "measure" else "pack",
                 "peak_source": peak_src + " hbm_gbs (copy bandwidth)",
                 "traffic_source": tsrc,
                 "algorithmic_bytes_per_launch": (mbytes if dominant == "measure"
                                                  else statistics.mean(pbytes))}
-    kernels = {"measure": {"ms": statistics.mean(measure_ms), "GBps": meas_gbs,
+    kernels = {measure_name: {"ms": statistics.mean(measure_ms), "GBps": meas_gbs,
                            "frac": meas_gbs / hbm, "bytes": mbytes},
                "select_and_readback": {"ms": statistics.mean(select_ms)},
                "pack": {"ms": statistics.mean(pack_ms), "GBps": pack_gbs, "frac": pack_gbs / hbm,
@@ -525,7 +571,7 @@ def run_ours(args):
             store.clear()
             if i >= max(1, args.warmup):
                 e_recs.append(r)
-                e_bytes.append(mbytes + pack_bytes(r["mask"], payload, wbytes))
+                e_bytes.append(mbytes + pack_bytes(r["mask"], payload, wbytes, fused_commit=not fused))
         e_s = sum(r["host_s"] for r in e_recs)
         d2h = statistics.mean(r["nbytes"] for r in e_recs)
         e2e = {"value": sum(e_bytes) / e_s / 1e9, "unit": "GB/s", "h2d_bytes_per_step": 0,
@@ -548,14 +594,20 @@ def run_ours(args):
         "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": statistics.mean(step_ms), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": "%s (%s, %d layers, %d params)" % (wl.name, shape.name, shape.nlayers,
-                                                               shape.numel),
+        "config": {"workload": "%s (%s, %d layers, %d params)%s" % (
+                       wl.name, shape.name, shape.nlayers, shape.numel,
+                       ", fused AdamW step + drift, fp32 master weights, bf16 gradients, "
+                       "lr %g" % FUSED_HP[0] if fused else ""),
                    "tau": tau, "max_staleness": K,
-                   "l2": ("inputs larger than L2 (%.1f GB read per measure)" % (mbytes / 1e9)
+                   "l2": ("inputs larger than L2 (%.1f GB %s per step)"
+                          % (mbytes / 1e9, "moved by the fused step" if fused else "read by the measure")
                           if flush is None else "L2 flushed before every step (%d MiB written; "
                           "%.1f MB read per measure)" % (flush.numel() >> 20, mbytes / 1e6)),
-                   "inputs": "bf16 weights and snapshot, fp32 Adam "
-                   "moments; arithmetic fp32 with fp64 combine", "parallelism": "dp%d" % world},
+                   "inputs": ("fp32 master weights, bf16 gradients and model copy, fp32 Adam moments, "
+                              "no snapshot; AdamW in fp32, drift sums fp32 with fp64 combine"
+                              if fused else "bf16 weights and snapshot, fp32 Adam moments; "
+                              "arithmetic fp32 with fp64 combine"),
+                   "parallelism": "dp%d" % world},
         "decision_ms_p50": statistics.median(decision_ms),
         "decision_ms_p99": float(np.percentile(decision_ms, 99)),
         "selected_fraction": frac_sel,

@@ -295,8 +295,8 @@ lc_status lc_register_optimizer(lc_ctx* ctx, const lc_optim_segment* segs, int32
  * Eq. 2).  step = t >= 1 is also the bias-correction count.  fp32
  * arithmetic, one rounding per operation in this order: p *= 1 - lr*wd;
  * m = beta1*m + (1-beta1)*g; v = beta2*v + (1-beta2)*(g*g);
- * p -= lr * ((m / (1-beta1^t)) / (sqrt(v / (1-beta2^t)) + eps)); the fp32
- * constants are formed in binary64 and rounded once.  Asynchronous.
+ * v_hat = v * (1/(1-beta2^t)); p -= (m * (lr/(1-beta1^t))) / (sqrt(v_hat) + eps);
+ * the fp32 constants are formed in binary64 and rounded once.  Asynchronous.
  * Errors: STATE (no optimizer registered, or a step is open), INVALID_ARG. */
 lc_status lc_adamw_step_measure(lc_ctx* ctx, int64_t step, const lc_adamw_hparams* hp);
 

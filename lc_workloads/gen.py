@@ -40,6 +40,8 @@ class SyntheticState:
 
     master=False keeps no fp32 master copy (a smaller footprint for kernel
     captures): the drift is then rounded into W at every step.
+    snapshot=False allocates no reference snapshot R (the fused optimizer
+    path measures the update itself).
     alloc: "separate" -- one allocation per tensor (16-byte aligned);
            "flat"     -- one buffer per kind, tensors back to back, so a
                          tensor after an odd-sized one starts misaligned;
@@ -48,7 +50,7 @@ class SyntheticState:
     """
 
     def __init__(self, shape, device="cuda", seed=0, alloc="separate", moments=True,
-                 dtypes=None, moments_mask=None, master=True):
+                 dtypes=None, moments_mask=None, master=True, snapshot=True):
         self.shape = shape
         self.device = torch.device(device)
         self.seed = int(seed)
@@ -59,6 +61,7 @@ class SyntheticState:
         self.has_moments = ([bool(moments)] * nt if moments_mask is None else
                             [bool(moments) and bool(x) for x in moments_mask])
         self.master = bool(master)
+        self.snapshot = bool(snapshot)
         self.W, self.R, self.M, self.m, self.v = [], [], [], [], []
         self._allocate()
         self.init()
@@ -84,7 +87,8 @@ class SyntheticState:
         if self.alloc == "separate":
             for k, t in enumerate(self.specs):
                 self.W.append(torch.empty(t.numel, dtype=self._tdtype(k), device=dev))
-                self.R.append(torch.empty(t.numel, dtype=self._tdtype(k), device=dev))
+                self.R.append(torch.empty(t.numel, dtype=self._tdtype(k), device=dev)
+                              if self.snapshot else None)
                 self.M.append(torch.empty(t.numel, dtype=torch.float32, device=dev)
                               if self.master else None)
                 mo = self.has_moments[k]
@@ -139,7 +143,8 @@ class SyntheticState:
                     self.W[k].copy_(self.M[k])
                 else:
                     self.W[k].normal_(0.0, 0.02, generator=g)
-                self.R[k].copy_(self.W[k])
+                if self.R[k] is not None:
+                    self.R[k].copy_(self.W[k])
                 self._draw_moments(0, k)
 
     def _draw_moments(self, step, k):

@@ -234,7 +234,9 @@ void lco_composite_pick(int32_t nversions, const int32_t* v_layer,
  *   m  <- beta1*m + (1-beta1)*g                 first moment
  *   v  <- beta2*v + (1-beta2)*g*g               second moment
  *   p  <- p - lr * (m/(1-beta1^t)) / (sqrt(v/(1-beta2^t)) + eps)
- * in binary32, the precision of the optimizer state, one rounding per
+ * in binary32, the precision of the optimizer state, with the two bias
+ * corrections folded into constants: v_hat = v * (1/(1-beta2^t)) and
+ * step = (m * (lr/(1-beta1^t))) / (sqrt(v_hat) + eps); one rounding per
  * operation in exactly this order.
  * ---------------------------------------------------------------------- */
 void lco_adamw_constants(const lco_adamw* hp, int64_t t, float out[9])
@@ -244,10 +246,10 @@ void lco_adamw_constants(const lco_adamw* hp, int64_t t, float out[9])
     out[2] = (float)(1.0 - hp->beta1);
     out[3] = (float)hp->beta2;
     out[4] = (float)(1.0 - hp->beta2);
-    out[5] = (float)(1.0 - pow(hp->beta1, (double)t));
-    out[6] = (float)(1.0 - pow(hp->beta2, (double)t));
-    out[7] = (float)hp->lr;
-    out[8] = (float)hp->eps;
+    out[5] = (float)(hp->lr / (1.0 - pow(hp->beta1, (double)t)));
+    out[6] = (float)(1.0 / (1.0 - pow(hp->beta2, (double)t)));
+    out[7] = (float)hp->eps;
+    out[8] = 0.0f;
 }
 
 uint16_t lco_bf16_round(float f)
@@ -269,7 +271,7 @@ void lco_adamw_step(const lco_adamw* hp, int64_t t, int64_t n, float* p, float* 
     float c[9];
     lco_adamw_constants(hp, t, c);
     const float decay = c[0], b1 = c[1], omb1 = c[2], b2 = c[3], omb2 = c[4];
-    const float bc1 = c[5], bc2 = c[6], lr = c[7], eps = c[8];
+    const float step_size = c[5], rbc2 = c[6], eps = c[7];
     double d_sum = 0.0, a_sum = 0.0;
     for (int64_t i = 0; i < n; ++i) {
         float g;
@@ -289,12 +291,11 @@ void lco_adamw_step(const lco_adamw* hp, int64_t t, int64_t n, float* p, float* 
         const float v1a = b2 * v[i];
         const float v1b = omb2 * gg;
         const float v_new = v1a + v1b;
-        const float m_hat = m_new / bc1;
-        const float v_hat = v_new / bc2;
+        const float v_hat = v_new * rbc2;
         const float root = sqrtf(v_hat);
         const float denom = root + eps;
-        const float step_dir = m_hat / denom;
-        const float step = lr * step_dir;
+        const float m_scaled = m_new * step_size;
+        const float step = m_scaled / denom;
         const float p_new = p_decayed - step;
         p[i] = p_new;
         m[i] = m_new;

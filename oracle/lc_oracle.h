@@ -96,8 +96,8 @@ typedef struct {
 
 /* fp32 constants of one AdamW step at step count t >= 1: out[0] = 1 - lr*wd,
  * out[1] = beta1, out[2] = 1 - beta1, out[3] = beta2, out[4] = 1 - beta2,
- * out[5] = 1 - beta1^t, out[6] = 1 - beta2^t, out[7] = lr, out[8] = eps;
- * each formed in binary64 and rounded once to binary32. */
+ * out[5] = lr / (1 - beta1^t), out[6] = 1 / (1 - beta2^t), out[7] = eps,
+ * out[8] = 0; each formed in binary64 and rounded once to binary32. */
 void lco_adamw_constants(const lco_adamw* hp, int64_t t, float out[9]);
 
 /* One AdamW step (decoupled weight decay) on n fp32 parameters in place,

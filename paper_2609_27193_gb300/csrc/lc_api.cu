@@ -676,9 +676,8 @@ extern "C" lc_status lc_adamw_step_measure(lc_ctx* ctx, int64_t step, const lc_a
     c.omb1 = float(1.0 - hp->beta1);
     c.b2 = float(hp->beta2);
     c.omb2 = float(1.0 - hp->beta2);
-    c.bc1 = float(1.0 - std::pow(hp->beta1, double(step)));
-    c.bc2 = float(1.0 - std::pow(hp->beta2, double(step)));
-    c.lr = float(hp->lr);
+    c.step_size = float(hp->lr / (1.0 - std::pow(hp->beta1, double(step))));
+    c.rbc2 = float(1.0 / (1.0 - std::pow(hp->beta2, double(step))));
     c.eps = float(hp->eps);
     DeviceGuard g(ctx->device);
     LC_CUDA(launch_adamw_measure(ctx->mp, ctx->d_opt, c, ctx->measure_grid, ctx->stream));

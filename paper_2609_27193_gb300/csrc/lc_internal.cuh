@@ -158,8 +158,9 @@ struct AdamConsts {
     float decay;           // 1 - lr*wd
     float b1, omb1;        // beta1, 1 - beta1
     float b2, omb2;        // beta2, 1 - beta2
-    float bc1, bc2;        // 1 - beta1^t, 1 - beta2^t
-    float lr, eps;
+    float step_size;       // lr / (1 - beta1^t)
+    float rbc2;            // 1 / (1 - beta2^t)
+    float eps;
 };
 
 // Launchers (return the launch error, if any).

@@ -54,8 +54,10 @@ MUTATIONS = [
      ["test_composite_pick_equals_replay", "test_crash_before_durable_uses_previous_version"]),
     ("composite-first-not-latest", "v_step[i] >= v_step[pick_out[l]]", "0",
      ["test_composite_pick_equals_replay", "test_composite_equals_latest_persisted_versions"]),
-    ("adamw-no-bias-correction", "const float m_hat = m_new / bc1;", "const float m_hat = m_new;",
+    ("adamw-no-second-bias-correction", "const float v_hat = v_new * rbc2;", "const float v_hat = v_new;",
      ["test_adamw_hand_cases", "test_constant_gradient_closed_form"]),
+    ("adamw-no-first-bias-correction", "out[5] = (float)(hp->lr / (1.0 - pow(hp->beta1, (double)t)));",
+     "out[5] = (float)hp->lr;", ["test_adamw_hand_cases", "test_constant_gradient_closed_form"]),
     ("adamw-second-moment-linear", "const float gg = g * g;", "const float gg = g;",
      ["test_adamw_hand_cases", "test_matches_binary64_adamw_within_fp32_rounding"]),
     ("adamw-decay-dropped", "const float p_decayed = p_old * decay;", "const float p_decayed = p_old;",
