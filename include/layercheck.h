@@ -260,6 +260,44 @@ lc_status lc_layer_block_bytes(const lc_ctx* ctx, int32_t layer, uint64_t* out);
 /* Library-side work counters of the context. */
 lc_status lc_get_counters(const lc_ctx* ctx, lc_counters* out);
 
+/* --- steps without a host round trip ------------------------------------ */
+
+/* One whole step -- measure (Eq. 1), select (Eq. 2-4, §3.3), pack of the
+ * persisted layers' full state (§3.1) into dst, snapshot commit -- enqueued
+ * on the context's stream with no host synchronization: the pack reads its
+ * size from device memory.  dst: device or pinned host memory (16-byte
+ * aligned; a pinned host buffer receives the stream directly over the host
+ * link), dst_capacity bytes.  If the step's stream would exceed
+ * dst_capacity, nothing is persisted and every layer keeps the
+ * not-persisted update (its drift stays accumulated); lc_step_wait then
+ * returns LC_ERR_CAPACITY.  Up to 4 steps may be in flight; the decision
+ * of each is read with lc_step_wait.  Requires snapshots (lc_measure's
+ * rules).  Errors: STATE (a step open, 4 in flight, no snapshot),
+ * INVALID_ARG, CUDA. */
+lc_status lc_step_async(lc_ctx* ctx, int64_t step, double tau, int32_t max_staleness,
+                        void* dst, uint64_t dst_capacity);
+
+/* Waits (bounded) for step `step` of lc_step_async or lc_step_graph_launch
+ * and returns its decision like lc_select (host arrays nullable); also
+ * updates lc_last_select_info / lc_last_select_offsets.
+ * Errors: NOT_FOUND (no such step in flight), CAPACITY (the step persisted
+ * nothing, see lc_step_async), TIMEOUT, CUDA. */
+lc_status lc_step_wait(lc_ctx* ctx, int64_t step, int32_t timeout_ms, uint8_t* mask_out,
+                       double* u_out, uint64_t* bytes_out);
+
+/* Captures the sequence of lc_step_async once as a CUDA graph with fixed
+ * tau, max_staleness and destination; the step number then comes from a
+ * device counter (previous step + 1).  Replaces an earlier graph of this
+ * context.  Errors: STATE, INVALID_ARG, CUDA. */
+lc_status lc_step_graph_create(lc_ctx* ctx, double tau, int32_t max_staleness, void* dst,
+                               uint64_t dst_capacity);
+
+/* Launches the captured step on the context's stream; *step_out (nullable)
+ * receives its step number.  The previous graph step must have been read
+ * with lc_step_wait.  Errors: STATE (no graph, or its last step not
+ * waited for), CUDA. */
+lc_status lc_step_graph_launch(lc_ctx* ctx, int64_t* step_out);
+
 /* --- fused optimizer step with the drift read off the update ------------ */
 
 /* Optimizer inputs of one segment, in the registration order of

@@ -165,6 +165,34 @@ class LayerCheck:
         check(self._lib.lc_last_select_offsets(self._ctx, o.ctypes.data))
         return o
 
+    def step_async(self, step, tau, max_staleness, dst):
+        """Enqueue a whole step (measure, select, pack into dst, commit) with
+        no host round trip; read the decision later with step_wait."""
+        check(self._lib.lc_step_async(self._ctx, int(step), float(tau), int(max_staleness),
+                                      C.c_void_p(dst.data_ptr()), int(dst.numel() * dst.element_size())))
+
+    def step_wait(self, step, timeout_ms=0):
+        """Decision of an asynchronous or graph step: (mask, u, bytes)."""
+        mask = np.zeros(self.nlayers, dtype=np.uint8)
+        u = np.zeros(self.nlayers, dtype=np.float64)
+        nbytes = C.c_uint64(0)
+        check(self._lib.lc_step_wait(self._ctx, int(step), int(timeout_ms), mask.ctypes.data,
+                                     u.ctypes.data, C.byref(nbytes)))
+        return mask, u, nbytes.value
+
+    def step_graph_create(self, tau, max_staleness, dst):
+        """Capture one step (fixed tau, S_max and destination) as a CUDA graph."""
+        self._keep.append(dst)
+        check(self._lib.lc_step_graph_create(self._ctx, float(tau), int(max_staleness),
+                                             C.c_void_p(dst.data_ptr()),
+                                             int(dst.numel() * dst.element_size())))
+
+    def step_graph_launch(self):
+        """Replay the captured step; returns its step number."""
+        s = C.c_int64(0)
+        check(self._lib.lc_step_graph_launch(self._ctx, C.byref(s)))
+        return s.value
+
     def pack_device(self, dst):
         """Gather into a uint8 CUDA (or pinned host) tensor."""
         check(self._lib.lc_pack_device(self._ctx, C.c_void_p(dst.data_ptr()),

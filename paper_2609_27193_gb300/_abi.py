@@ -93,6 +93,10 @@ SIGNATURES = {
     "lc_store_num_versions": (C.c_int64, [store_p]),
     "lc_store_get_version": (C.c_int, [store_p, C.c_int64, P(lc_version)]),
     "lc_store_plan": (C.c_int, [store_p, C.c_int64, C.c_void_p]),
+    "lc_step_async": (C.c_int, [ctx_p, C.c_int64, C.c_double, C.c_int32, C.c_void_p, C.c_uint64]),
+    "lc_step_wait": (C.c_int, [ctx_p, C.c_int64, C.c_int32, C.c_void_p, C.c_void_p, P(C.c_uint64)]),
+    "lc_step_graph_create": (C.c_int, [ctx_p, C.c_double, C.c_int32, C.c_void_p, C.c_uint64]),
+    "lc_step_graph_launch": (C.c_int, [ctx_p, P(C.c_int64)]),
     "lc_register_optimizer": (C.c_int, [ctx_p, P(lc_optim_segment), C.c_int32]),
     "lc_adamw_step_measure": (C.c_int, [ctx_p, C.c_int64, P(lc_adamw_hparams)]),
     "lc_measure_noalloc": (C.c_int, [C.c_int, C.c_void_p, P(lc_segment), C.c_int32, C.c_int32,

@@ -197,6 +197,19 @@ struct lc_ctx {
     std::vector<uint64_t> offsets;
     std::vector<PendingPack> pending;
     lc_counters counters{};
+
+    // device-driven steps: pinned decision blocks of steps still in flight
+    struct AsyncSlot {
+        uint8_t* host = nullptr;   // pinned copy of the decision block
+        cudaEvent_t done = nullptr;
+        int64_t step = -1;
+        bool busy = false;
+    };
+    static constexpr int kAsyncSlots = 4;
+    AsyncSlot slots[kAsyncSlots + 1];   // the last one belongs to the captured graph
+    cudaStream_t capture_stream = nullptr;
+    cudaGraphExec_t graph_exec = nullptr;
+    bool graph_mode_commit = false;
 };
 
 // ---------------------------------------------------------------------------
@@ -278,6 +291,12 @@ extern "C" void lc_destroy(lc_ctx* ctx) {
         }
     }
     for (auto& pp : ctx->pending) cudaEventDestroy(pp.done);
+    for (auto& sl : ctx->slots) {
+        if (sl.host) cudaFreeHost(sl.host);
+        if (sl.done) cudaEventDestroy(sl.done);
+    }
+    if (ctx->graph_exec) cudaGraphExecDestroy(ctx->graph_exec);
+    if (ctx->capture_stream) cudaStreamDestroy(ctx->capture_stream);
     cudaFree(ctx->d_tables);
     cudaFree(ctx->d_opt);
     cudaFree(ctx->d_staging);
@@ -495,6 +514,9 @@ extern "C" lc_status lc_register_layout(lc_ctx* ctx, const lc_segment* segs, int
     const size_t o_lwsec = tp.take(sizeof(int32_t) * nlayers);
     const size_t o_secs = tp.take(sizeof(SectionDev) * std::max(1, nsec));
     const size_t o_scratch = tp.take(sizeof(int64_t) * 3 * nlayers);
+    const size_t o_accsave = tp.take(sizeof(double) * nlayers);
+    const size_t o_tlsave = tp.take(sizeof(int64_t) * nlayers);
+    const size_t o_stepctr = tp.take(sizeof(int64_t));
     ctx->rl = result_layout(nlayers);
     const size_t o_result = tp.take(ctx->rl.total);
     const size_t o_pdesc = tp.take(sizeof(CopyDesc) * std::max(1, nsec));
@@ -503,6 +525,10 @@ extern "C" lc_status lc_register_layout(lc_ctx* ctx, const lc_segment* segs, int
     const size_t total = tp.size;
 
     std::vector<uint8_t> host(total, 0);
+    {
+        const int64_t before_first_step = -1;
+        std::memcpy(host.data() + o_stepctr, &before_first_step, sizeof before_first_step);
+    }
     auto put = [&](size_t off, const void* src, size_t n) { if (n) std::memcpy(host.data() + off, src, n); };
     put(o_segs, sd.data(), sizeof(SegDev) * nseg);
     put(o_ctav, cta_vec.data(), sizeof(int64_t) * (G + 1));
@@ -549,6 +575,11 @@ extern "C" lc_status lc_register_layout(lc_ctx* ctx, const lc_segment* segs, int
     sp.layer_wsec_count = reinterpret_cast<const int32_t*>(base + o_lwsec);
     sp.secs = reinterpret_cast<const SectionDev*>(base + o_secs);
     sp.layer_scratch = reinterpret_cast<int64_t*>(base + o_scratch);
+    sp.acc_save = reinterpret_cast<double*>(base + o_accsave);
+    sp.tl_save = reinterpret_cast<int64_t*>(base + o_tlsave);
+    sp.step_counter = reinterpret_cast<int64_t*>(base + o_stepctr);
+    sp.capacity = UINT64_MAX;
+    sp.step_from_counter = 0;
     sp.result = base + o_result;
     sp.pack_desc = reinterpret_cast<CopyDesc*>(base + o_pdesc);
     sp.commit_desc = reinterpret_cast<CopyDesc*>(base + o_cdesc);
@@ -731,7 +762,7 @@ extern "C" lc_status lc_select(lc_ctx* ctx, double tau, int32_t max_staleness, u
 
     ResultHeader h;
     std::memcpy(&h, ctx->h_result, sizeof h);
-    if (h.magic != kResultMagic || h.step != ctx->last_step)
+    if (h.magic != kResultMagic || h.step != ctx->last_step || h.status != kStatusOk)
         return fail(LC_ERR_CUDA, "lc_select: decision block is corrupt");
     const uint8_t* m = ctx->h_result + ctx->rl.mask_off;
     const double* u = reinterpret_cast<const double*>(ctx->h_result + ctx->rl.u_off);
@@ -785,6 +816,8 @@ lc_status launch_copy_range(lc_ctx* ctx, const CopyDesc* desc, int ndesc, int mo
     p.lo = lo;
     p.hi = hi;
     p.base = base;
+    p.ndesc_dev = nullptr;
+    p.hi_dev = nullptr;
     const uint64_t units = (hi - lo) >> 4;
     const int grid = int(std::max<uint64_t>(1, std::min<uint64_t>(uint64_t(ctx->copy_grid), units)));
     LC_CUDA(launch_copy(p, grid, s));
@@ -969,6 +1002,201 @@ extern "C" lc_status lc_wait_durable(lc_ctx* ctx, int64_t step, int32_t timeout_
 }
 
 // ---------------------------------------------------------------------------
+// device-driven steps (no host round trip) and their captured graph
+// ---------------------------------------------------------------------------
+namespace {
+
+lc_status ensure_slot_memory(lc_ctx* ctx, lc_ctx::AsyncSlot& sl) {
+    if (!sl.host) LC_CUDA(cudaHostAlloc(reinterpret_cast<void**>(&sl.host), ctx->rl.total, cudaHostAllocDefault));
+    if (!sl.done) LC_CUDA(cudaEventCreateWithFlags(&sl.done, cudaEventDisableTiming));
+    return LC_OK;
+}
+
+lc_status check_step_dst(lc_ctx* ctx, void* dst, uint64_t capacity) {
+    if (capacity > 0) {
+        if (!dst) return fail(LC_ERR_INVALID_ARG, "step: dst is NULL");
+        if (uintptr_t(dst) & 15) return fail(LC_ERR_INVALID_ARG, "step: dst must be 16-byte aligned");
+        LC_TRY(check_device_ptr(dst, ctx->device, "step dst", true));
+    }
+    if (ctx->snap_missing) return fail(LC_ERR_STATE, "step: a segment has no snapshot to measure against");
+    return LC_OK;
+}
+
+// Enqueues measure -> select -> pack -> commit -> decision readback on s.
+lc_status enqueue_step(lc_ctx* ctx, cudaStream_t s, int64_t step, bool step_from_counter, double tau,
+                       int32_t max_staleness, uint8_t* dst, uint64_t capacity, uint8_t* host_block) {
+    LC_CUDA(launch_measure(ctx->mp, ctx->measure_grid, ctx->cfg.mode == LC_DRIFT_ACCUMULATE, s));
+    SelectParams p = ctx->sp;
+    p.tau = tau;
+    p.max_staleness = max_staleness;
+    p.step = step;
+    p.step_from_counter = step_from_counter ? 1 : 0;
+    p.capacity = capacity;
+    LC_CUDA(launch_select(p, s));
+    const ResultHeader* hdr_dev = reinterpret_cast<const ResultHeader*>(ctx->d_result);
+    CopyParams c;
+    c.desc = ctx->d_pack_desc;
+    c.ndesc = 0;
+    c.mode = kGather;
+    c.lo = 0;
+    c.hi = 0;
+    c.base = dst;
+    c.ndesc_dev = &hdr_dev->n_pack_desc;
+    c.hi_dev = &hdr_dev->pack_bytes;
+    LC_CUDA(launch_copy(c, ctx->copy_grid, s));
+    int launches = 3;
+    if (ctx->cfg.mode == LC_DRIFT_SNAPSHOT && !ctx->cfg.fuse_commit) {
+        CopyParams k = c;
+        k.desc = ctx->d_commit_desc;
+        k.mode = kCopy;
+        k.base = nullptr;
+        k.ndesc_dev = &hdr_dev->n_commit_desc;
+        k.hi_dev = &hdr_dev->commit_work;
+        LC_CUDA(launch_copy(k, ctx->copy_grid, s));
+        launches += 1;
+    }
+    LC_CUDA(cudaMemcpyAsync(host_block, ctx->d_result, ctx->rl.total, cudaMemcpyDeviceToHost, s));
+    ctx->counters.kernel_launches += launches;
+    ctx->counters.measure_launches += 1;
+    ctx->counters.select_launches += 1;
+    ctx->counters.copy_launches += launches - 2;
+    ctx->counters.d2h_bytes += ctx->rl.total;
+    return LC_OK;
+}
+
+}  // namespace
+
+extern "C" lc_status lc_step_async(lc_ctx* ctx, int64_t step, double tau, int32_t max_staleness,
+                                   void* dst, uint64_t dst_capacity) {
+    g_err.clear();
+    if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_step_async: ctx is NULL");
+    if (ctx->state == kNew) return fail(LC_ERR_STATE, "lc_step_async: no layout registered");
+    if (step_open(ctx)) return fail(LC_ERR_STATE, "lc_step_async: a step is open");
+    if (step < 0 || step <= ctx->last_step)
+        return fail(LC_ERR_INVALID_ARG, "lc_step_async: step %lld must exceed the previous step %lld",
+                    (long long)step, (long long)ctx->last_step);
+    if (!std::isfinite(tau) || max_staleness < 0)
+        return fail(LC_ERR_INVALID_ARG, "lc_step_async: tau must be finite and max_staleness >= 0");
+    DeviceGuard g(ctx->device);
+    LC_TRY(check_step_dst(ctx, dst, dst_capacity));
+    int free_slot = -1;
+    for (int i = 0; i < lc_ctx::kAsyncSlots; ++i)
+        if (!ctx->slots[i].busy) { free_slot = i; break; }
+    if (free_slot < 0)
+        return fail(LC_ERR_STATE, "lc_step_async: %d steps in flight; call lc_step_wait", lc_ctx::kAsyncSlots);
+    lc_ctx::AsyncSlot& sl = ctx->slots[free_slot];
+    LC_TRY(ensure_slot_memory(ctx, sl));
+    LC_TRY(enqueue_step(ctx, ctx->stream, step, false, tau, max_staleness, static_cast<uint8_t*>(dst),
+                        dst_capacity, sl.host));
+    LC_CUDA(cudaEventRecord(sl.done, ctx->stream));
+    sl.step = step;
+    sl.busy = true;
+    ctx->last_step = step;
+    return LC_OK;
+}
+
+extern "C" lc_status lc_step_wait(lc_ctx* ctx, int64_t step, int32_t timeout_ms, uint8_t* mask_out,
+                                  double* u_out, uint64_t* bytes_out) {
+    g_err.clear();
+    if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_step_wait: ctx is NULL");
+    lc_ctx::AsyncSlot* sl = nullptr;
+    for (auto& s : ctx->slots)
+        if (s.busy && s.step == step) { sl = &s; break; }
+    if (!sl) return fail(LC_ERR_NOT_FOUND, "lc_step_wait: no step %lld in flight", (long long)step);
+    DeviceGuard g(ctx->device);
+    LC_TRY(wait_event(sl->done, timeout_ms > 0 ? timeout_ms : ctx->cfg.timeout_ms, "lc_step_wait"));
+    sl->busy = false;
+    ResultHeader h;
+    std::memcpy(&h, sl->host, sizeof h);
+    if (h.magic != kResultMagic || h.step != step)
+        return fail(LC_ERR_CUDA, "lc_step_wait: decision block of step %lld is corrupt", (long long)step);
+    const uint8_t* m = sl->host + ctx->rl.mask_off;
+    const double* u = reinterpret_cast<const double*>(sl->host + ctx->rl.u_off);
+    const uint64_t* o = reinterpret_cast<const uint64_t*>(sl->host + ctx->rl.off_off);
+    for (int32_t l = 0; l < ctx->nlayers; ++l) {
+        ctx->mask[l] = m[l];
+        ctx->offsets[l] = o[l];
+    }
+    if (mask_out) std::memcpy(mask_out, m, size_t(ctx->nlayers));
+    if (u_out) std::memcpy(u_out, u, sizeof(double) * size_t(ctx->nlayers));
+    if (bytes_out) *bytes_out = h.bytes;
+    ctx->hdr = h;
+    ctx->have_select = true;
+    if (h.status == kStatusCapacity)
+        return fail(LC_ERR_CAPACITY,
+                    "step %lld: the %llu-byte stream exceeded the destination; nothing was persisted",
+                    (long long)step, (unsigned long long)h.bytes);
+    return LC_OK;
+}
+
+extern "C" lc_status lc_step_graph_create(lc_ctx* ctx, double tau, int32_t max_staleness, void* dst,
+                                          uint64_t dst_capacity) {
+    g_err.clear();
+    if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_step_graph_create: ctx is NULL");
+    if (ctx->state == kNew) return fail(LC_ERR_STATE, "lc_step_graph_create: no layout registered");
+    if (step_open(ctx)) return fail(LC_ERR_STATE, "lc_step_graph_create: a step is open");
+    if (!std::isfinite(tau) || max_staleness < 0)
+        return fail(LC_ERR_INVALID_ARG, "lc_step_graph_create: tau must be finite and max_staleness >= 0");
+    DeviceGuard g(ctx->device);
+    LC_TRY(check_step_dst(ctx, dst, dst_capacity));
+    lc_ctx::AsyncSlot& sl = ctx->slots[lc_ctx::kAsyncSlots];
+    if (sl.busy) return fail(LC_ERR_STATE, "lc_step_graph_create: the graph's last step was not waited for");
+    LC_TRY(ensure_slot_memory(ctx, sl));
+    if (!ctx->capture_stream) LC_CUDA(cudaStreamCreateWithFlags(&ctx->capture_stream, cudaStreamNonBlocking));
+    if (ctx->graph_exec) {
+        cudaGraphExecDestroy(ctx->graph_exec);
+        ctx->graph_exec = nullptr;
+    }
+    const lc_counters before = ctx->counters;
+    LC_CUDA(cudaStreamBeginCapture(ctx->capture_stream, cudaStreamCaptureModeThreadLocal));
+    lc_status rc = enqueue_step(ctx, ctx->capture_stream, 0, true, tau, max_staleness,
+                                static_cast<uint8_t*>(dst), dst_capacity, sl.host);
+    cudaGraph_t graph = nullptr;
+    const cudaError_t e = cudaStreamEndCapture(ctx->capture_stream, &graph);
+    ctx->counters = before;      // capture runs nothing; launches count when the graph is replayed
+    if (rc != LC_OK) {
+        if (graph) cudaGraphDestroy(graph);
+        return rc;
+    }
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return fail(LC_ERR_CUDA, "lc_step_graph_create: capture failed: %s", cudaGetErrorString(e));
+    }
+    const cudaError_t ei = cudaGraphInstantiate(&ctx->graph_exec, graph, 0);
+    cudaGraphDestroy(graph);
+    if (ei != cudaSuccess) {
+        cudaGetLastError();
+        ctx->graph_exec = nullptr;
+        return fail(LC_ERR_CUDA, "lc_step_graph_create: instantiate failed: %s", cudaGetErrorString(ei));
+    }
+    ctx->graph_mode_commit = ctx->cfg.mode == LC_DRIFT_SNAPSHOT && !ctx->cfg.fuse_commit;
+    return LC_OK;
+}
+
+extern "C" lc_status lc_step_graph_launch(lc_ctx* ctx, int64_t* step_out) {
+    g_err.clear();
+    if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_step_graph_launch: ctx is NULL");
+    if (!ctx->graph_exec) return fail(LC_ERR_STATE, "lc_step_graph_launch: no graph (lc_step_graph_create)");
+    if (step_open(ctx)) return fail(LC_ERR_STATE, "lc_step_graph_launch: a step is open");
+    lc_ctx::AsyncSlot& sl = ctx->slots[lc_ctx::kAsyncSlots];
+    if (sl.busy) return fail(LC_ERR_STATE, "lc_step_graph_launch: wait for step %lld first", (long long)sl.step);
+    DeviceGuard g(ctx->device);
+    LC_CUDA(cudaGraphLaunch(ctx->graph_exec, ctx->stream));
+    LC_CUDA(cudaEventRecord(sl.done, ctx->stream));
+    const int launches = ctx->graph_mode_commit ? 4 : 3;
+    ctx->counters.kernel_launches += launches;
+    ctx->counters.measure_launches += 1;
+    ctx->counters.select_launches += 1;
+    ctx->counters.copy_launches += launches - 2;
+    ctx->counters.d2h_bytes += ctx->rl.total;
+    ctx->last_step += 1;
+    sl.step = ctx->last_step;
+    sl.busy = true;
+    if (step_out) *step_out = ctx->last_step;
+    return LC_OK;
+}
+
+// ---------------------------------------------------------------------------
 // restore (§3.5, Eq. 8)
 // ---------------------------------------------------------------------------
 extern "C" lc_status lc_restore(lc_ctx* ctx, lc_store* st, int64_t t_fail, int64_t* layer_steps_out) {
@@ -1054,6 +1282,8 @@ extern "C" lc_status lc_restore(lc_ctx* ctx, lc_store* st, int64_t t_fail, int64
                                         cudaMemcpyHostToDevice, ctx->stream);
         if (e == cudaSuccess)
             e = cudaMemcpyAsync(ctx->sp.delta, zeros.data(), sizeof(double) * N, cudaMemcpyHostToDevice, ctx->stream);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(ctx->sp.step_counter, &t_fail, sizeof t_fail, cudaMemcpyHostToDevice, ctx->stream);
         if (e == cudaSuccess) e = cudaEventRecord(ev_desc, ctx->stream);
         if (e != cudaSuccess) {
             cudaGetLastError();

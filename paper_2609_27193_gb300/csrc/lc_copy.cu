@@ -136,7 +136,11 @@ __device__ void copy_entry(const CopyParams& p, const CopyDesc& d, uint64_t a, u
     }
 }
 
-__global__ void __launch_bounds__(kCopyThreads) copy_kernel(const CopyParams p) {
+__global__ void __launch_bounds__(kCopyThreads) copy_kernel(CopyParams p) {
+    if (p.ndesc_dev) {           // sizes decided on the device by the select kernel
+        p.ndesc = *p.ndesc_dev;
+        p.hi = p.lo + *p.hi_dev;
+    }
     // CTA ranges in granules of LC_COPY_ALIGN_BYTES (the last one ragged)
     constexpr uint64_t kGran = LC_COPY_ALIGN_BYTES / 16;
     const uint64_t units = (p.hi - p.lo) >> 4;

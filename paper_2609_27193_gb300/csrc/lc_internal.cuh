@@ -79,6 +79,10 @@ struct CopyParams {
     int32_t mode;
     uint64_t lo, hi;     // work range of this launch; lo and hi multiples of 16
     uint8_t* base;       // stream buffer holding work offset lo (GATHER / SCATTER)
+    // Device-driven launches (no host round trip): when set, the entry count
+    // and the end of the range are read from device memory at kernel start.
+    const int32_t* ndesc_dev;
+    const uint64_t* hi_dev;
 };
 
 // A section of a layer's packed block (one segment's W, exp_avg or exp_avg_sq).
@@ -103,9 +107,12 @@ struct ResultHeader {
     int64_t max_staleness;
     double weighted_staleness;
     uint32_t magic;
-    uint32_t reserved;
+    uint32_t status;           // kStatusOk, or kStatusCapacity: nothing persisted
+    uint64_t pack_bytes;       // bytes the pack moves: `bytes`, or 0 after kStatusCapacity
 };
 constexpr uint32_t kResultMagic = 0x4C43534Cu;
+constexpr uint32_t kStatusOk = 0;
+constexpr uint32_t kStatusCapacity = 1;
 
 struct ResultLayout {
     size_t mask_off, u_off, off_off, total;
@@ -134,9 +141,14 @@ struct SelectParams {
     uint8_t* result;                 // decision block (device)
     CopyDesc* pack_desc;             // [nsec]
     CopyDesc* commit_desc;           // [nseg]
+    double* acc_save;                // [nlayers] the step's accumulated drift (for a rollback)
+    int64_t* tl_save;                // [nlayers] t_l before the step
+    int64_t* step_counter;           // last step decided on the device
     double tau;
     double eps_w;
-    int64_t step;
+    int64_t step;                    // the step, unless step_from_counter
+    uint64_t capacity;               // bytes the destination holds (UINT64_MAX: unchecked)
+    int32_t step_from_counter;       // 1: step = *step_counter + 1 (captured graphs)
     int32_t max_staleness;
     int32_t nlayers;
     int32_t mode;                    // lc_drift_mode

@@ -7,7 +7,10 @@
 // finite; it resets Delta_l and sets t_l = t for persisted layers.  It then
 // assigns each persisted layer its offset in the packed stream (layers
 // ascending) and writes the copy lists of the pack and of the snapshot
-// commit, so the host never builds them.
+// commit, so the host never builds them.  If the stream would not fit the
+// destination, it persists nothing and restores every layer's state to the
+// not-persisted update (the drift stays accumulated).  The step comes from
+// the host, or from a device counter when the step runs as a CUDA graph.
 #include "lc_internal.cuh"
 
 namespace lc {
@@ -22,22 +25,31 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectPara
     int64_t* scratch = p.layer_scratch;
 
     __shared__ int s_nonfinite;
-    if (threadIdx.x == 0) s_nonfinite = 0;
+    __shared__ int64_t s_step;
+    __shared__ uint32_t s_status;
+    if (threadIdx.x == 0) {
+        s_nonfinite = 0;
+        s_step = p.step_from_counter ? *p.step_counter + 1 : p.step;
+        *p.step_counter = s_step;
+    }
     __syncthreads();
+    const int64_t step = s_step;
 
     for (int l = threadIdx.x; l < p.nlayers; l += blockDim.x) {
         const double d = p.sums[3 * l], a = p.sums[3 * l + 1], n = p.sums[3 * l + 2];
         const double u = (d / n) / (a / n + p.eps_w);                     // Eq. 1
         const double acc = p.mode == 1 ? p.delta[l] + u : u;              // Eq. 2
         const double threshold = p.tau * p.tau_mult[l];
-        const int64_t staleness = p.step - p.t_last[l];
+        const int64_t staleness = step - p.t_last[l];
         const bool nonfinite = !isfinite(acc);
         const bool persist = nonfinite || acc >= threshold                // Eq. 3
                              || staleness >= int64_t(p.max_staleness);     // §3.3
         if (nonfinite) atomicAdd(&s_nonfinite, 1);
+        p.acc_save[l] = acc;
+        p.tl_save[l] = p.t_last[l];
         if (persist) {                                                     // Eq. 4
             p.delta[l] = 0.0;
-            p.t_last[l] = p.step;
+            p.t_last[l] = step;
         } else {
             p.delta[l] = acc;
         }
@@ -52,7 +64,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectPara
         int64_t mx = 0;
         double num = 0.0, den = 0.0;
         for (int l = 0; l < p.nlayers; ++l) {
-            const int64_t st = p.step - p.t_last[l];
+            const int64_t st = step - p.t_last[l];
             mx = st > mx ? st : mx;
             num = __dadd_rn(num, __dmul_rn(double(p.layer_numel[l]), double(st)));
             den = __dadd_rn(den, double(p.layer_numel[l]));
@@ -73,20 +85,32 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectPara
                 off[l] = 0;
             }
         }
-        hdr->step = p.step;
+        // a stream larger than the destination persists nothing this step
+        const bool fits = run <= p.capacity;
+        hdr->step = step;
         hdr->n_selected = nsel;
         hdr->n_nonfinite = s_nonfinite;
         hdr->bytes = run;
-        hdr->n_pack_desc = nsec;
-        hdr->n_commit_desc = ncommit;
-        hdr->commit_work = commit_work;
+        hdr->n_pack_desc = fits ? nsec : 0;
+        hdr->n_commit_desc = fits ? ncommit : 0;
+        hdr->commit_work = fits ? commit_work : 0;
         hdr->max_staleness = mx;
         hdr->weighted_staleness = den > 0.0 ? num / den : 0.0;
         hdr->magic = kResultMagic;
-        hdr->reserved = 0;
+        hdr->status = fits ? kStatusOk : kStatusCapacity;
+        hdr->pack_bytes = fits ? run : 0;
+        s_status = hdr->status;
     }
     __syncthreads();
 
+    if (s_status != kStatusOk) {
+        // roll back to "nothing persisted": the drift stays accumulated
+        for (int l = threadIdx.x; l < p.nlayers; l += blockDim.x) {
+            p.delta[l] = p.acc_save[l];
+            p.t_last[l] = p.tl_save[l];
+        }
+        return;
+    }
     const bool fused = p.fuse_commit != 0 && p.mode == 0;
     for (int l = threadIdx.x; l < p.nlayers; l += blockDim.x) {
         if (!mask[l]) continue;
