@@ -53,9 +53,10 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--shape-blocks", type=int, default=0,
                     help="keep only the first N transformer blocks (small case for kernel captures)")
-    ap.add_argument("--path", choices=["scan", "fused"], default="scan",
+    ap.add_argument("--path", choices=["scan", "fused", "graph"], default="scan",
                     help="scan: measure against the snapshot (default); fused: AdamW step with "
-                         "the drift read off the update, fp32 master weights")
+                         "the drift read off the update, fp32 master weights; graph: the scan "
+                         "step replayed as one captured CUDA graph with no host round trip")
     ap.add_argument("--lean", action="store_true",
                     help="no fp32 master weights in the generator (small case for kernel captures)")
     return ap.parse_args()
@@ -442,6 +443,25 @@ def run_ours(args):
             grads[k].copy_(tmp.add_(float(grad_bias[spec.layer])).mul_(1e-3))
             del tmp
 
+    graph = args.path == "graph"
+    overflow = []
+
+    def graph_step(t, ev, h0):
+        ev[0].record(side)
+        s_t = lc.step_graph_launch()     # the graph numbers its own steps (from 0)
+        for e in ev[1:]:
+            e.record(side)
+        try:
+            mask, u, nbytes = lc.step_wait(s_t)
+        except P.LCError as err:
+            if err.status != 5:
+                raise
+            overflow.append(t)
+            mask, u, nbytes = np.zeros(shape.nlayers, np.uint8), None, 0
+        h1 = time.perf_counter()
+        main.wait_stream(side)
+        return dict(ev=ev, decision_s=h1 - h0, host_s=h1 - h0, mask=mask, nbytes=nbytes)
+
     def step(t, mode, store=None):
         new_inputs(t)
         if flush is not None:
@@ -456,6 +476,8 @@ def run_ours(args):
                     torch.matmul(a, b, out=c)
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
         h0 = time.perf_counter()
+        if graph:
+            return graph_step(t, ev, h0)
         ev[0].record(side)
         if fused:
             lc.adamw_step_measure(t, FUSED_HP[0], FUSED_HP[1], FUSED_HP[2], FUSED_HP[3], FUSED_HP[4])
@@ -481,6 +503,9 @@ def run_ours(args):
         h2 = time.perf_counter()
         main.wait_stream(side)
         return dict(ev=ev, decision_s=h1 - h0, host_s=h2 - h0, mask=mask, nbytes=nbytes)
+
+    if graph:
+        lc.step_graph_create(tau, K, dst)
 
     # ---- device-resident phase: the `value` --------------------------------
     t = 0
@@ -549,6 +574,18 @@ def run_ours(args):
                "select_and_readback": {"ms": statistics.mean(select_ms)},
                "pack": {"ms": statistics.mean(pack_ms), "GBps": pack_gbs, "frac": pack_gbs / hbm,
                         "bytes": statistics.mean(pbytes)}}
+    if graph:
+        # one replay covers measure, select, pack and the decision readback:
+        # only the whole step is timed, and its bytes are measure + pack
+        g_bytes = mbytes + statistics.mean(pbytes)
+        g_gbs = g_bytes / (statistics.mean(step_ms) / 1e3) / 1e9
+        kernels = {"graph_step": {"ms": statistics.mean(step_ms), "GBps": g_gbs, "frac": g_gbs / hbm,
+                                  "bytes": g_bytes, "launches_per_step": 3}}
+        roofline = {"bound": "hbm", "achieved": g_gbs, "peak": hbm, "unit": "GB/s",
+                    "frac": g_gbs / hbm, "traffic": None,
+                    "kernel": "graph step (measure, select, pack, commit)",
+                    "peak_source": peak_src + " hbm_gbs (copy bandwidth)", "traffic_source": None,
+                    "algorithmic_bytes_per_launch": g_bytes}
 
     # ---- end to end through the pinned host store --------------------------
     e2e = None
@@ -562,13 +599,21 @@ def run_ours(args):
         except OSError:
             pass
         cap = full if avail == 0 else min(full, int(avail * 0.6))
-        store = P.Store(lc, capacity_bytes=cap)
+        if graph:
+            # the replayed pack writes straight into pinned host memory
+            store = None
+            hcap = min(cap, int(max(r["nbytes"] for r in recs) * 1.5) + (64 << 20))
+            hostdst = torch.empty(hcap, dtype=torch.uint8, pin_memory=True)
+            lc.step_graph_create(tau, K, hostdst)
+        else:
+            store = P.Store(lc, capacity_bytes=cap)
         link = d2h_link_probe(torch, dev)
         e_recs, e_bytes = [], []
         for i in range(max(1, args.warmup) + args.steps):
             t += 1
             r = step(t, "store", store)
-            store.clear()
+            if store is not None:
+                store.clear()
             if i >= max(1, args.warmup):
                 e_recs.append(r)
                 e_bytes.append(mbytes + pack_bytes(r["mask"], payload, wbytes, fused_commit=not fused))
@@ -577,12 +622,15 @@ def run_ours(args):
         e2e = {"value": sum(e_bytes) / e_s / 1e9, "unit": "GB/s", "h2d_bytes_per_step": 0,
                "d2h_bytes_per_step": int(d2h),
                "ms_per_step": 1e3 * e_s / len(e_recs),
-               "d2h_GBps": d2h / (statistics.mean(r["host_s"] - r["decision_s"] for r in e_recs)) / 1e9,
+               "d2h_GBps": d2h / (statistics.mean((r["host_s"] - r["decision_s"]) if not graph
+                                                  else r["host_s"] for r in e_recs)) / 1e9,
                "d2h_link_GBps_measured": link,
                "note": "weights, snapshot and moments are device-resident training state; the "
                        "step's only host traffic is the decision block and the persisted "
-                       "layers copied into the pinned store"}
-        store.close()
+                       "layers copied into %s" % ("pinned host memory by the replayed graph's pack"
+                                                  if graph else "the pinned store")}
+        if store is not None:
+            store.close()
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -614,6 +662,7 @@ def run_ours(args):
         "persisted_bytes_per_step": statistics.mean(r["nbytes"] for r in recs),
         "roofline": roofline, "kernels": kernels, "e2e": e2e, "cpu_baseline": cpu,
         "gpu_launches": int(c1["kernel_launches"] - c0["kernel_launches"]),
+        "capacity_overflow_steps": overflow,
         "clocks": clk, "timed_wall_s_with_input_generation": wall, "setup_s": setup_s,
     }
     if rank == 0:
