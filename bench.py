@@ -57,6 +57,9 @@ def parse_args():
                     help="scan: measure against the snapshot (default); fused: AdamW step with "
                          "the drift read off the update, fp32 master weights; graph: the scan "
                          "step replayed as one captured CUDA graph with no host round trip")
+    ap.add_argument("--copy-engine", choices=["threads", "bulk"], default="threads",
+                    help="threads: per-thread 16-byte vector copies (default); bulk: the "
+                         "bulk-copy engine through shared memory when every buffer is device memory")
     ap.add_argument("--lean", action="store_true",
                     help="no fp32 master weights in the generator (small case for kernel captures)")
     return ap.parse_args()
@@ -93,7 +96,8 @@ def kernel_source_sha(files):
 
 KERNEL_FILES = {"measure": ["lc_measure.cu", "lc_reduce.cuh", "lc_internal.cuh"],
                 "fused_adamw": ["lc_adamw.cu", "lc_reduce.cuh", "lc_internal.cuh"],
-                "pack": ["lc_copy.cu", "lc_internal.cuh"]}
+                "pack": ["lc_copy.cu", "lc_internal.cuh"],
+                "pack_bulk": ["lc_copy.cu", "lc_internal.cuh"]}
 
 
 def profiled_traffic(kernel, workload, persisted_bytes=None):
@@ -393,7 +397,8 @@ def run_ours(args):
     if fused:
         # fp32 master weights are the optimizer's parameters; the bf16 W is the
         # model copy the step refreshes; no snapshot is kept
-        lc = P.LayerCheck(device=local, stream=side, mode=P.LC_DRIFT_ACCUMULATE)
+        lc = P.LayerCheck(device=local, stream=side, mode=P.LC_DRIFT_ACCUMULATE,
+                          copy_engine=args.copy_engine)
         lc.register_layout([P.segment(t.layer, st.M[k], None, st.m[k], st.v[k])
                             for k, t in enumerate(shape.tensors)], shape.nlayers)
         grads = [torch.empty(t.numel, dtype=torch.bfloat16, device=dev) for t in shape.tensors]
@@ -401,7 +406,7 @@ def run_ours(args):
         # per-layer gradient bias: layers with consistent gradients move faster
         grad_bias = gen.u_shape(shape.nlayers, 2.0, 0.05, 0.3, np.random.default_rng(wl.seed + 7))
     else:
-        lc = P.LayerCheck(device=local, stream=side)
+        lc = P.LayerCheck(device=local, stream=side, copy_engine=args.copy_engine)
         lc.register_layout([P.segment(t.layer, st.W[k], st.R[k], st.m[k], st.v[k])
                             for k, t in enumerate(shape.tensors)], shape.nlayers)
     sums = None
@@ -555,7 +560,8 @@ def run_ours(args):
     dominant = "measure" if sum(measure_ms) >= sum(pack_ms) else "pack"
     measure_name = "fused_adamw" if fused else "measure"
     mean_persisted = statistics.mean(r["nbytes"] for r in recs)
-    traffic, tsrc = profiled_traffic(measure_name if dominant == "measure" else "pack",
+    pack_name = "pack" if args.copy_engine == "threads" else "pack_bulk"
+    traffic, tsrc = profiled_traffic(measure_name if dominant == "measure" else pack_name,
                                      args.workload, mean_persisted if dominant == "pack" else None)
     if fused and dominant == "pack":
         traffic, tsrc = None, None       # the pack profile is of bf16 weights
@@ -655,6 +661,7 @@ def run_ours(args):
                               "no snapshot; AdamW in fp32, drift sums fp32 with fp64 combine"
                               if fused else "bf16 weights and snapshot, fp32 Adam moments; "
                               "arithmetic fp32 with fp64 combine"),
+                   "copy_engine": args.copy_engine,
                    "parallelism": "dp%d" % world},
         "decision_ms_p50": statistics.median(decision_ms),
         "decision_ms_p99": float(np.percentile(decision_ms, 99)),
@@ -662,6 +669,7 @@ def run_ours(args):
         "persisted_bytes_per_step": statistics.mean(r["nbytes"] for r in recs),
         "roofline": roofline, "kernels": kernels, "e2e": e2e, "cpu_baseline": cpu,
         "gpu_launches": int(c1["kernel_launches"] - c0["kernel_launches"]),
+        "bulk_copy_launches": int(c1["bulk_copy_launches"] - c0["bulk_copy_launches"]),
         "capacity_overflow_steps": overflow,
         "clocks": clk, "timed_wall_s_with_input_generation": wall, "setup_s": setup_s,
     }

@@ -71,6 +71,24 @@ typedef enum { LC_BF16 = 0, LC_F32 = 1 } lc_dtype;
  *                      R <- W for every layer and Eq. 2 sums u_l over steps. */
 typedef enum { LC_DRIFT_SNAPSHOT = 0, LC_DRIFT_ACCUMULATE = 1 } lc_drift_mode;
 
+/* Kernel that moves packed, committed and restored bytes (the bytes are the
+ * same either way).
+ * LC_COPY_THREADS: every thread loads and stores 16-byte vectors (default;
+ *                  the faster one on the packs measured so far).
+ * LC_COPY_BULK   : the bulk-copy engine (cp.async.bulk through shared
+ *                  memory) whenever every address of the copy is device
+ *                  memory -- segments, staging ring and destination -- else
+ *                  as LC_COPY_THREADS. */
+typedef enum { LC_COPY_THREADS = 0, LC_COPY_BULK = 1 } lc_copy_engine;
+
+/* LC_DEBUG_BULK_STALL: every bulk-engine copy launch waits for 16 bytes that
+ * never arrive, once per CTA.  The engine's bounded wait (1 s) runs out, the
+ * launch sets the context's copy-fault word and returns without finishing
+ * its bytes, and the next call that checks the word (lc_select,
+ * lc_wait_durable, lc_step_wait, lc_restore) fails with LC_ERR_TIMEOUT for
+ * good.  It exists to test that path; it faults and hangs nothing. */
+#define LC_DEBUG_BULK_STALL 1
+
 /* One parameter tensor ("segment") of a layer (§2.2: embed_tokens, each
  * transformer block, the final norm and lm_head are the layers; a layer
  * may hold several tensors).
@@ -107,6 +125,8 @@ typedef struct {
     int32_t timeout_ms;      /* bound of every host wait (default 60000)          */
     uint64_t staging_bytes;  /* device staging ring used by lc_pack_async and
                                 lc_restore, split in two slots (default 512 MiB) */
+    int32_t copy_engine;     /* lc_copy_engine (default LC_COPY_THREADS)         */
+    int32_t debug_flags;     /* 0, or LC_DEBUG_BULK_STALL (tests only)           */
 } lc_config;
 
 typedef struct lc_ctx lc_ctx;
@@ -141,6 +161,7 @@ typedef struct {
     int64_t copy_launches;       /* pack / commit / restore copy kernels        */
     uint64_t d2h_bytes;          /* bytes copied device -> host by the library  */
     uint64_t h2d_bytes;          /* bytes copied host -> device by the library  */
+    int64_t bulk_copy_launches;  /* copy launches that ran on the bulk engine   */
 } lc_counters;
 
 /* Fills cfg with the defaults listed in lc_config. */
@@ -364,6 +385,70 @@ lc_status lc_store_get_version(const lc_store* store, int64_t index, lc_version*
  * layer l with the largest step <= t_fail (the newer record on a tie), or
  * -1.  Returns NOT_FOUND if some layer has none. */
 lc_status lc_store_plan(const lc_store* store, int64_t t_fail, int64_t* pick_out);
+
+/* --- file tier of the store: §3.5 metadata-driven recovery -------------- *
+ * A checkpoint directory holds two append-only files.
+ *   blocks.lcb   : packed layer blocks (the §3.1 layout of lc_pack_*), each
+ *                  starting on a 4096-byte boundary.
+ *   manifest.lcm : a 64-byte header, then one 64-byte record per block.
+ * All integers are little-endian.  Header: "LCMH", format 1 (u32), nlayers
+ * (i32), layout CRC (u32: CRC-32C of the nlayers block sizes as u64), zeros,
+ * and at byte 60 the CRC-32C of bytes [0, 60).  Record: "LCVR", layer (i32),
+ * step (i64), offset in blocks.lcb (u64), bytes (u64), CRC-32C of the block
+ * (u32), layout CRC (u32), zeros, and at byte 60 the CRC-32C of [0, 60).
+ * A block is written (and synced, if asked) before its record, so a record
+ * never names a block that is not there; the log ends at the first short or
+ * invalid record (a torn append), which the next append overwrites.  The
+ * recovery reads the records only -- the metadata -- to choose, per layer,
+ * the newest version at or before the failure step (§3.5), and then reads
+ * just those blocks, checking each against its CRC. */
+
+/* CRC-32C (Castagnoli, reflected polynomial 0x82F63B78, initial value and
+ * final XOR 0xFFFFFFFF) of data[0, nbytes), continuing from `crc` (0 to
+ * start; crc32c(B, crc32c(A, 0)) is the CRC of A followed by B).  Host
+ * memory; large inputs are split over the host's cores. */
+uint32_t lc_crc32c(const void* data, uint64_t nbytes, uint32_t crc);
+
+/* Appends to directory `dir` (created if missing) every durable version of
+ * `store` whose (layer, step) the manifest does not hold yet, in version
+ * order.  sync != 0: each block and each record is fdatasync'd before the
+ * next write.  bytes_written (nullable): block bytes appended.  Call it from
+ * the thread that drives the store's context, between steps.
+ * Errors: INVALID_ARG (dir holds another layout, or is unusable), STATE
+ * (the manifest's header is corrupt). */
+lc_status lc_store_persist_dir(lc_store* store, const char* dir, int32_t sync, uint64_t* bytes_written);
+
+/* §3.5 / Eq. 8 from a checkpoint directory: for every layer of ctx's layout
+ * the version with the largest step <= t_fail (the later record on a tie)
+ * whose record and block CRCs check out; a version whose block fails its CRC
+ * is passed over for the next older one.  Reads only those blocks, into a
+ * new log store (*out, one durable version per layer, owned by the caller:
+ * lc_store_destroy) that lc_restore(ctx, *out, t_fail, ...) then scatters
+ * onto the device.  layer_steps_out: host, nlayers (nullable).
+ * Errors: NOT_FOUND (a layer has no intact version <= t_fail), INVALID_ARG
+ * (another layout, no manifest), STATE, OOM. */
+lc_status lc_store_load_dir(lc_ctx* ctx, const char* dir, int64_t t_fail, lc_store** out,
+                            int64_t* layer_steps_out);
+
+/* One manifest record as read back. */
+typedef struct {
+    int32_t layer;
+    int32_t intact;          /* block CRC checked and equal (verify_blocks), else 1 */
+    int64_t step;
+    uint64_t offset;         /* in blocks.lcb */
+    uint64_t bytes;
+    uint32_t block_crc;
+    uint32_t layout_crc;
+} lc_manifest_record;
+
+/* Reads the manifest of `dir` without a GPU.  out (nullable) receives up to
+ * cap valid records in file order; *n_out = the number of valid records;
+ * *nlayers_out and *layout_crc_out from the header; *torn_out = 1 if the log
+ * ends in a short or invalid record.  verify_blocks != 0 reads every block
+ * and sets `intact` from its CRC.  Any out pointer may be NULL.
+ * Errors: INVALID_ARG (no manifest), STATE (corrupt header). */
+lc_status lc_manifest_read(const char* dir, int32_t verify_blocks, lc_manifest_record* out, int64_t cap,
+                           int64_t* n_out, int32_t* nlayers_out, uint32_t* layout_crc_out, int32_t* torn_out);
 
 /* --- the measure without any device allocation -------------------------- */
 

@@ -11,20 +11,49 @@ C ABI of include/layercheck.h (the raw functions keep their C names in
 ``paper_2609_27193_gb300._abi``).  There is no CPU fallback.
 """
 import ctypes as C
+import os
 
 import numpy as np
 
 from . import _abi
-from ._abi import (LC_BF16, LC_DRIFT_ACCUMULATE, LC_DRIFT_SNAPSHOT, LC_F32, LCError, check,
-                   lc_config, lc_counters, lc_segment, lc_select_info, lc_version)
+from ._abi import (LC_BF16, LC_COPY_BULK, LC_COPY_THREADS, LC_DEBUG_BULK_STALL,
+                   LC_DRIFT_ACCUMULATE, LC_DRIFT_SNAPSHOT, LC_F32, LCError, check, lc_config,
+                   lc_counters, lc_segment, lc_select_info, lc_version)
 
 __all__ = ["LayerCheck", "Store", "LCError", "LC_BF16", "LC_F32", "LC_DRIFT_SNAPSHOT",
-           "LC_DRIFT_ACCUMULATE", "library", "segment"]
+           "LC_DRIFT_ACCUMULATE", "LC_DEBUG_BULK_STALL", "library", "segment", "crc32c",
+           "manifest_read"]
 
 
 def library():
     """The loaded ctypes library (raises ImportError when not built)."""
     return _abi.load()
+
+
+def crc32c(data, crc=0):
+    """CRC-32C of a bytes-like object or contiguous numpy array (host)."""
+    buf = np.ascontiguousarray(np.frombuffer(data, dtype=np.uint8) if not isinstance(data, np.ndarray)
+                               else data.view(np.uint8).reshape(-1))
+    return int(library().lc_crc32c(buf.ctypes.data, buf.size, int(crc)))
+
+
+def manifest_read(path, verify_blocks=True):
+    """The valid records of a checkpoint directory's manifest (no GPU):
+    (records as dicts in file order, nlayers, layout CRC, torn tail?)."""
+    from ._abi import lc_manifest_record
+    lib = library()
+    n = C.c_int64(0)
+    nl = C.c_int32(0)
+    lay = C.c_uint32(0)
+    torn = C.c_int32(0)
+    check(lib.lc_manifest_read(os.fsencode(path), 0, None, 0, C.byref(n), C.byref(nl), C.byref(lay),
+                               C.byref(torn)))
+    recs = (lc_manifest_record * max(1, n.value))()
+    check(lib.lc_manifest_read(os.fsencode(path), int(bool(verify_blocks)), recs, n.value, C.byref(n),
+                               C.byref(nl), C.byref(lay), C.byref(torn)))
+    out = [{name: getattr(recs[i], name) for name, _ in lc_manifest_record._fields_}
+           for i in range(n.value)]
+    return out, nl.value, lay.value, bool(torn.value)
 
 
 def _dtype_code(t):
@@ -55,13 +84,19 @@ class LayerCheck:
     """One library context on one device and one CUDA stream."""
 
     def __init__(self, device=0, stream=None, eps_w=1e-8, mode=LC_DRIFT_SNAPSHOT,
-                 pack_align=256, fuse_commit=True, timeout_ms=60000, staging_bytes=512 << 20):
+                 pack_align=256, fuse_commit=True, timeout_ms=60000, staging_bytes=512 << 20,
+                 copy_engine="threads", debug_flags=0):
         lib = library()
         cfg = lc_config()
         lib.lc_config_default(C.byref(cfg))
         cfg.eps_w, cfg.mode, cfg.pack_align = float(eps_w), int(mode), int(pack_align)
         cfg.fuse_commit, cfg.timeout_ms = int(bool(fuse_commit)), int(timeout_ms)
         cfg.staging_bytes = int(staging_bytes)
+        engines = {"threads": LC_COPY_THREADS, "bulk": LC_COPY_BULK}
+        if copy_engine not in engines:
+            raise ValueError("copy_engine must be one of %s" % sorted(engines))
+        cfg.copy_engine = engines[copy_engine]
+        cfg.debug_flags = int(debug_flags)
         if stream is None:
             import torch
             stream = torch.cuda.current_stream(device)
@@ -212,6 +247,16 @@ class LayerCheck:
         check(self._lib.lc_restore(self._ctx, store.handle, int(t_fail), steps.ctypes.data))
         return steps
 
+    def load_dir(self, path, t_fail):
+        """§3.5 recovery from a checkpoint directory: each layer's newest
+        intact version at or before t_fail, read into a new Store (one
+        version per layer) for restore().  Returns (store, steps)."""
+        steps = np.zeros(self.nlayers, dtype=np.int64)
+        h = C.c_void_p()
+        check(self._lib.lc_store_load_dir(self._ctx, os.fsencode(path), int(t_fail), C.byref(h),
+                                          steps.ctypes.data))
+        return Store._adopt(h, self.nlayers), steps
+
     def layer_block_bytes(self, layer):
         b = C.c_uint64(0)
         check(self._lib.lc_layer_block_bytes(self._ctx, int(layer), C.byref(b)))
@@ -234,9 +279,22 @@ class Store:
         self._h = h
         self.nlayers = lc.nlayers
 
+    @classmethod
+    def _adopt(cls, handle, nlayers):
+        st = cls.__new__(cls)
+        st._lib, st._h, st.nlayers = library(), handle, nlayers
+        return st
+
     @property
     def handle(self):
         return self._h
+
+    def persist_dir(self, path, sync=False):
+        """Appends the durable versions the directory does not hold yet
+        (file tier, format in layercheck.h); returns the block bytes written."""
+        n = C.c_uint64(0)
+        check(self._lib.lc_store_persist_dir(self._h, os.fsencode(path), int(bool(sync)), C.byref(n)))
+        return n.value
 
     def close(self):
         if getattr(self, "_h", None) and self._h.value:

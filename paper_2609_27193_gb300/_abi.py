@@ -22,6 +22,8 @@ STATUS_NAMES = {0: "LC_OK", 1: "LC_ERR_INVALID_ARG", 2: "LC_ERR_STATE", 3: "LC_E
 
 LC_BF16, LC_F32 = 0, 1
 LC_DRIFT_SNAPSHOT, LC_DRIFT_ACCUMULATE = 0, 1
+LC_COPY_THREADS, LC_COPY_BULK = 0, 1
+LC_DEBUG_BULK_STALL = 1
 
 
 class lc_segment(C.Structure):
@@ -33,7 +35,8 @@ class lc_segment(C.Structure):
 class lc_config(C.Structure):
     _fields_ = [("eps_w", C.c_double), ("mode", C.c_int32), ("pack_align", C.c_int32),
                 ("fuse_commit", C.c_int32), ("timeout_ms", C.c_int32),
-                ("staging_bytes", C.c_uint64)]
+                ("staging_bytes", C.c_uint64), ("copy_engine", C.c_int32),
+                ("debug_flags", C.c_int32)]
 
 
 class lc_select_info(C.Structure):
@@ -60,7 +63,14 @@ class lc_adamw_hparams(C.Structure):
 class lc_counters(C.Structure):
     _fields_ = [("kernel_launches", C.c_int64), ("measure_launches", C.c_int64),
                 ("select_launches", C.c_int64), ("copy_launches", C.c_int64),
-                ("d2h_bytes", C.c_uint64), ("h2d_bytes", C.c_uint64)]
+                ("d2h_bytes", C.c_uint64), ("h2d_bytes", C.c_uint64),
+                ("bulk_copy_launches", C.c_int64)]
+
+
+class lc_manifest_record(C.Structure):
+    _fields_ = [("layer", C.c_int32), ("intact", C.c_int32), ("step", C.c_int64),
+                ("offset", C.c_uint64), ("bytes", C.c_uint64), ("block_crc", C.c_uint32),
+                ("layout_crc", C.c_uint32)]
 
 
 ctx_p = C.c_void_p
@@ -101,6 +111,11 @@ SIGNATURES = {
     "lc_adamw_step_measure": (C.c_int, [ctx_p, C.c_int64, P(lc_adamw_hparams)]),
     "lc_measure_noalloc": (C.c_int, [C.c_int, C.c_void_p, P(lc_segment), C.c_int32, C.c_int32,
                                      C.c_void_p]),
+    "lc_crc32c": (C.c_uint32, [C.c_void_p, C.c_uint64, C.c_uint32]),
+    "lc_store_persist_dir": (C.c_int, [store_p, C.c_char_p, C.c_int32, P(C.c_uint64)]),
+    "lc_store_load_dir": (C.c_int, [ctx_p, C.c_char_p, C.c_int64, P(store_p), C.c_void_p]),
+    "lc_manifest_read": (C.c_int, [C.c_char_p, C.c_int32, P(lc_manifest_record), C.c_int64,
+                                   P(C.c_int64), P(C.c_int32), P(C.c_uint32), P(C.c_int32)]),
 }
 
 # limits of lc_measure_noalloc (include/layercheck.h)

@@ -6,6 +6,7 @@
 // the kernels of lc_measure.cu, lc_select.cu and lc_copy.cu on the caller's
 // stream.  No compute happens here: every step of the path runs on the GPU.
 #include "layercheck.h"
+#include "lc_host.h"
 #include "lc_internal.cuh"
 
 #include <algorithm>
@@ -166,6 +167,10 @@ struct lc_ctx {
     std::vector<int32_t> sec_seg;          // segment (measure order) of each section
     std::vector<int32_t> sec_part;         // 0 = W, 1 = exp_avg, 2 = exp_avg_sq
     int measure_grid = 0, copy_grid = 0, nslots = 0;
+    int bulk_grid = 0;                     // CTAs of a bulk-engine copy launch
+    bool bulk_sources = false;             // every registered array is device memory
+    uint32_t* h_fault = nullptr;           // pinned, mapped: a bulk copy gave up waiting
+    uint32_t* d_fault = nullptr;           // its device address
     bool any_write_ref = false;
     std::vector<int32_t> order;            // measure position -> registration index
     bool snap_missing = false;             // some segment has no snapshot
@@ -209,8 +214,48 @@ struct lc_ctx {
     AsyncSlot slots[kAsyncSlots + 1];   // the last one belongs to the captured graph
     cudaStream_t capture_stream = nullptr;
     cudaGraphExec_t graph_exec = nullptr;
-    bool graph_mode_commit = false;
+    lc_counters graph_delta{};             // what one replay of the graph launches
 };
+
+namespace {
+
+// True for memory of cudaMalloc (not managed, not host): the only kind the
+// bulk-copy engine is given.
+bool plain_device(const void* p) {
+    cudaPointerAttributes a;
+    if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return a.type == cudaMemoryTypeDevice;
+}
+
+// A bulk copy whose bounded wait ran out leaves the word set for good: the
+// bytes of that copy (and so every later checkpoint) are not to be trusted.
+lc_status check_copy_fault(const lc_ctx* ctx, const char* what) {
+    if (ctx->h_fault && *reinterpret_cast<volatile const uint32_t*>(ctx->h_fault))
+        return fail(LC_ERR_TIMEOUT, "%s: a bulk-engine copy gave up waiting for its loads", what);
+    return LC_OK;
+}
+
+// Engine and grid of a copy launch whose stream-side buffer is `base`
+// (nullptr when the launch has none).
+bool use_bulk(const lc_ctx* ctx, const void* base) {
+    return ctx->cfg.copy_engine == LC_COPY_BULK && ctx->bulk_sources && (!base || plain_device(base));
+}
+
+cudaError_t launch_copy_engine(lc_ctx* ctx, CopyParams p, bool bulk, uint64_t units, cudaStream_t s) {
+    p.fault = ctx->d_fault;
+    p.stall_first = (ctx->cfg.debug_flags & LC_DEBUG_BULK_STALL) ? 1 : 0;
+    const uint64_t cap = uint64_t(bulk ? ctx->bulk_grid : ctx->copy_grid);
+    const int grid = int(std::max<uint64_t>(1, std::min<uint64_t>(cap, units)));
+    ctx->counters.kernel_launches += 1;
+    ctx->counters.copy_launches += 1;
+    if (bulk) ctx->counters.bulk_copy_launches += 1;
+    return bulk ? launch_copy_bulk(p, grid, s) : launch_copy(p, grid, s);
+}
+
+}  // namespace
 
 // ---------------------------------------------------------------------------
 // config, errors, create, destroy
@@ -247,6 +292,10 @@ extern "C" lc_status lc_create(lc_ctx** out, int device, void* cuda_stream, cons
     if (c.timeout_ms <= 0) return fail(LC_ERR_INVALID_ARG, "lc_create: timeout_ms must be > 0");
     if (c.staging_bytes < (2u << 20))
         return fail(LC_ERR_INVALID_ARG, "lc_create: staging_bytes must be >= 2 MiB");
+    if (c.copy_engine != LC_COPY_THREADS && c.copy_engine != LC_COPY_BULK)
+        return fail(LC_ERR_INVALID_ARG, "lc_create: unknown copy engine %d", c.copy_engine);
+    if (c.debug_flags & ~LC_DEBUG_BULK_STALL)
+        return fail(LC_ERR_INVALID_ARG, "lc_create: unknown debug flags 0x%x", unsigned(c.debug_flags));
     int ndev = 0;
     LC_CUDA(cudaGetDeviceCount(&ndev));
     if (device < 0 || device >= ndev)
@@ -269,11 +318,20 @@ extern "C" lc_status lc_create(lc_ctx** out, int device, void* cuda_stream, cons
         e = cudaEventCreateWithFlags(&ctx->ev_slot_free[i], cudaEventDisableTiming);
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->ev_slot_filled[i], cudaEventDisableTiming);
     }
+    if (e == cudaSuccess)
+        e = cudaHostAlloc(reinterpret_cast<void**>(&ctx->h_fault), sizeof(uint32_t), cudaHostAllocMapped);
+    if (e == cudaSuccess) {
+        *ctx->h_fault = 0;
+        e = cudaHostGetDevicePointer(reinterpret_cast<void**>(&ctx->d_fault), ctx->h_fault, 0);
+    }
+    int bocc = 0;
+    if (e == cudaSuccess) e = copy_bulk_prepare(&bocc);
     if (e != cudaSuccess) {
         cudaGetLastError();
         lc_destroy(ctx);
         return fail(LC_ERR_CUDA, "lc_create: %s", cudaGetErrorString(e));
     }
+    ctx->bulk_grid = ctx->sms * std::max(1, bocc);
     *out = ctx;
     return LC_OK;
 }
@@ -301,6 +359,7 @@ extern "C" void lc_destroy(lc_ctx* ctx) {
     cudaFree(ctx->d_opt);
     cudaFree(ctx->d_staging);
     if (ctx->h_result) cudaFreeHost(ctx->h_result);
+    if (ctx->h_fault) cudaFreeHost(ctx->h_fault);
     if (ctx->ev_result) cudaEventDestroy(ctx->ev_result);
     for (int i = 0; i < 2; ++i) {
         if (ctx->ev_slot_free[i]) cudaEventDestroy(ctx->ev_slot_free[i]);
@@ -374,6 +433,12 @@ extern "C" lc_status lc_register_layout(lc_ctx* ctx, const lc_segment* segs, int
     }
     for (int32_t l = 0; l < nlayers; ++l)
         if (per_layer[l] == 0) return fail(LC_ERR_INVALID_ARG, "layer %d has no segment", l);
+    bool all_device = true;
+    for (int32_t i = 0; i < nseg && all_device; ++i) {
+        const lc_segment& s = segs[i];
+        all_device = plain_device(s.w) && (!s.snap || plain_device(s.snap)) &&
+                     (!s.exp_avg || (plain_device(s.exp_avg) && plain_device(s.exp_avg_sq)));
+    }
     std::vector<double> mult(nlayers, 1.0);
     if (tau_mult) {
         for (int32_t l = 0; l < nlayers; ++l) {
@@ -389,6 +454,7 @@ extern "C" lc_status lc_register_layout(lc_ctx* ctx, const lc_segment* segs, int
     std::stable_sort(order.begin(), order.end(),
                      [&](int32_t a, int32_t b) { return segs[a].layer < segs[b].layer; });
     ctx->nseg = nseg;
+    ctx->bulk_sources = all_device;
     ctx->nlayers = nlayers;
     ctx->segs.resize(nseg);
     for (int32_t i = 0; i < nseg; ++i) ctx->segs[i] = segs[order[i]];
@@ -759,6 +825,7 @@ extern "C" lc_status lc_select(lc_ctx* ctx, double tau, int32_t max_staleness, u
     ctx->counters.d2h_bytes += ctx->rl.total;
     LC_CUDA(cudaEventRecord(ctx->ev_result, ctx->stream));
     LC_TRY(wait_event(ctx->ev_result, ctx->cfg.timeout_ms, "lc_select"));
+    LC_TRY(check_copy_fault(ctx, "lc_select"));
 
     ResultHeader h;
     std::memcpy(&h, ctx->h_result, sizeof h);
@@ -818,11 +885,7 @@ lc_status launch_copy_range(lc_ctx* ctx, const CopyDesc* desc, int ndesc, int mo
     p.base = base;
     p.ndesc_dev = nullptr;
     p.hi_dev = nullptr;
-    const uint64_t units = (hi - lo) >> 4;
-    const int grid = int(std::max<uint64_t>(1, std::min<uint64_t>(uint64_t(ctx->copy_grid), units)));
-    LC_CUDA(launch_copy(p, grid, s));
-    ctx->counters.kernel_launches += 1;
-    ctx->counters.copy_launches += 1;
+    LC_CUDA(launch_copy_engine(ctx, p, use_bulk(ctx, base), (hi - lo) >> 4, s));
     return LC_OK;
 }
 
@@ -987,6 +1050,7 @@ extern "C" lc_status lc_wait_durable(lc_ctx* ctx, int64_t step, int32_t timeout_
         if (pp.step != step) { ++i; continue; }
         found = true;
         LC_TRY(wait_event(pp.done, tmo, "lc_wait_durable"));
+        LC_TRY(check_copy_fault(ctx, "lc_wait_durable"));
         {
             std::lock_guard<std::mutex> lk(g_store_mu);
             if (g_live_stores.count(pp.store)) {
@@ -1043,8 +1107,8 @@ lc_status enqueue_step(lc_ctx* ctx, cudaStream_t s, int64_t step, bool step_from
     c.base = dst;
     c.ndesc_dev = &hdr_dev->n_pack_desc;
     c.hi_dev = &hdr_dev->pack_bytes;
-    LC_CUDA(launch_copy(c, ctx->copy_grid, s));
-    int launches = 3;
+    // sizes are decided on the device: full grids, idle CTAs return at once
+    LC_CUDA(launch_copy_engine(ctx, c, use_bulk(ctx, dst), UINT64_MAX, s));
     if (ctx->cfg.mode == LC_DRIFT_SNAPSHOT && !ctx->cfg.fuse_commit) {
         CopyParams k = c;
         k.desc = ctx->d_commit_desc;
@@ -1052,14 +1116,12 @@ lc_status enqueue_step(lc_ctx* ctx, cudaStream_t s, int64_t step, bool step_from
         k.base = nullptr;
         k.ndesc_dev = &hdr_dev->n_commit_desc;
         k.hi_dev = &hdr_dev->commit_work;
-        LC_CUDA(launch_copy(k, ctx->copy_grid, s));
-        launches += 1;
+        LC_CUDA(launch_copy_engine(ctx, k, use_bulk(ctx, nullptr), UINT64_MAX, s));
     }
     LC_CUDA(cudaMemcpyAsync(host_block, ctx->d_result, ctx->rl.total, cudaMemcpyDeviceToHost, s));
-    ctx->counters.kernel_launches += launches;
+    ctx->counters.kernel_launches += 2;
     ctx->counters.measure_launches += 1;
     ctx->counters.select_launches += 1;
-    ctx->counters.copy_launches += launches - 2;
     ctx->counters.d2h_bytes += ctx->rl.total;
     return LC_OK;
 }
@@ -1106,6 +1168,7 @@ extern "C" lc_status lc_step_wait(lc_ctx* ctx, int64_t step, int32_t timeout_ms,
     DeviceGuard g(ctx->device);
     LC_TRY(wait_event(sl->done, timeout_ms > 0 ? timeout_ms : ctx->cfg.timeout_ms, "lc_step_wait"));
     sl->busy = false;
+    LC_TRY(check_copy_fault(ctx, "lc_step_wait"));
     ResultHeader h;
     std::memcpy(&h, sl->host, sizeof h);
     if (h.magic != kResultMagic || h.step != step)
@@ -1153,7 +1216,15 @@ extern "C" lc_status lc_step_graph_create(lc_ctx* ctx, double tau, int32_t max_s
                                 static_cast<uint8_t*>(dst), dst_capacity, sl.host);
     cudaGraph_t graph = nullptr;
     const cudaError_t e = cudaStreamEndCapture(ctx->capture_stream, &graph);
+    const lc_counters after = ctx->counters;
     ctx->counters = before;      // capture runs nothing; launches count when the graph is replayed
+    ctx->graph_delta = lc_counters{};
+    ctx->graph_delta.kernel_launches = after.kernel_launches - before.kernel_launches;
+    ctx->graph_delta.measure_launches = after.measure_launches - before.measure_launches;
+    ctx->graph_delta.select_launches = after.select_launches - before.select_launches;
+    ctx->graph_delta.copy_launches = after.copy_launches - before.copy_launches;
+    ctx->graph_delta.bulk_copy_launches = after.bulk_copy_launches - before.bulk_copy_launches;
+    ctx->graph_delta.d2h_bytes = after.d2h_bytes - before.d2h_bytes;
     if (rc != LC_OK) {
         if (graph) cudaGraphDestroy(graph);
         return rc;
@@ -1169,7 +1240,6 @@ extern "C" lc_status lc_step_graph_create(lc_ctx* ctx, double tau, int32_t max_s
         ctx->graph_exec = nullptr;
         return fail(LC_ERR_CUDA, "lc_step_graph_create: instantiate failed: %s", cudaGetErrorString(ei));
     }
-    ctx->graph_mode_commit = ctx->cfg.mode == LC_DRIFT_SNAPSHOT && !ctx->cfg.fuse_commit;
     return LC_OK;
 }
 
@@ -1183,12 +1253,13 @@ extern "C" lc_status lc_step_graph_launch(lc_ctx* ctx, int64_t* step_out) {
     DeviceGuard g(ctx->device);
     LC_CUDA(cudaGraphLaunch(ctx->graph_exec, ctx->stream));
     LC_CUDA(cudaEventRecord(sl.done, ctx->stream));
-    const int launches = ctx->graph_mode_commit ? 4 : 3;
-    ctx->counters.kernel_launches += launches;
-    ctx->counters.measure_launches += 1;
-    ctx->counters.select_launches += 1;
-    ctx->counters.copy_launches += launches - 2;
-    ctx->counters.d2h_bytes += ctx->rl.total;
+    const lc_counters& d = ctx->graph_delta;
+    ctx->counters.kernel_launches += d.kernel_launches;
+    ctx->counters.measure_launches += d.measure_launches;
+    ctx->counters.select_launches += d.select_launches;
+    ctx->counters.copy_launches += d.copy_launches;
+    ctx->counters.bulk_copy_launches += d.bulk_copy_launches;
+    ctx->counters.d2h_bytes += d.d2h_bytes;
     ctx->last_step += 1;
     sl.step = ctx->last_step;
     sl.busy = true;
@@ -1293,6 +1364,7 @@ extern "C" lc_status lc_restore(lc_ctx* ctx, lc_store* st, int64_t t_fail, int64
         }
     }
     cudaEventDestroy(ev_desc);
+    if (rc == LC_OK) rc = check_copy_fault(ctx, "lc_restore");
     if (rc != LC_OK) return rc;
     if (layer_steps_out) std::memcpy(layer_steps_out, steps.data(), sizeof(int64_t) * N);
     ctx->last_step = t_fail;
@@ -1435,4 +1507,36 @@ extern "C" lc_status lc_store_plan(const lc_store* st, int64_t t_fail, int64_t* 
             return fail(LC_ERR_NOT_FOUND, "lc_store_plan: layer %d has no durable version at or before step %lld",
                         l, (long long)t_fail);
     return LC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// host internals used by the file tier (lc_files.cu)
+// ---------------------------------------------------------------------------
+int32_t lc::ctx_nlayers(const lc_ctx* ctx) { return ctx->nlayers; }
+int32_t lc::store_nlayers(const lc_store* st) { return st->nlayers; }
+const uint64_t* lc::store_layer_bytes(const lc_store* st) { return st->layer_bytes.data(); }
+
+uint8_t* lc::store_append(lc_store* st, int32_t layer, int64_t* index_out) {
+    if (st->per_layer != 0 || layer < 0 || layer >= st->nlayers) return nullptr;
+    const uint64_t bytes = st->layer_bytes[size_t(layer)];
+    if (st->top + bytes > st->capacity) return nullptr;
+    st->versions.push_back({st->next_id++, layer, 1, -1, st->top, bytes, -1});
+    uint8_t* p = st->arena + st->top;
+    st->top += bytes;
+    if (index_out) *index_out = int64_t(st->versions.size()) - 1;
+    return p;
+}
+
+void lc::store_set_step(lc_store* st, int64_t index, int64_t step) {
+    if (index >= 0 && size_t(index) < st->versions.size()) st->versions[size_t(index)].step = step;
+}
+
+lc_status lc::fail_status(lc_status st, const char* fmt, ...) {
+    char buf[1024];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_err = buf;
+    return st;
 }

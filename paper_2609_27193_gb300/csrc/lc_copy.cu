@@ -1,6 +1,8 @@
-// lc_copy.cu -- the byte-moving kernel behind the pack (§3.1 full layer
+// lc_copy.cu -- the byte-moving kernels behind the pack (§3.1 full layer
 // state into one contiguous stream), the snapshot commit and the restore
-// scatter (§3.5).
+// scatter (§3.5): copy_kernel (every thread loads and stores 16-byte
+// vectors) and copy_bulk_kernel (the payload goes through shared memory on
+// the bulk-copy engine; used when every address is device memory).
 //
 // A launch covers the work range [lo, hi) of a descriptor list whose
 // entries tile a linear work space (lc_internal.cuh).  The range is cut into
@@ -56,23 +58,25 @@ __device__ __forceinline__ void st_v4(void* p, uint4 v) {
 #endif
 }
 
-// 16-byte vectors [v0, v1) of an entry, LC_COPY_UNROLL loads in flight per thread.
+// 16-byte vectors [v0, v1) of an entry, LC_COPY_UNROLL loads in flight per
+// thread; thread tid of NT workers.
+template <int NT>
 __device__ __forceinline__ void copy_vec(const uint8_t* src, uint8_t* dst, uint8_t* dst2,
-                                         uint64_t v0, uint64_t v1) {
+                                         uint64_t v0, uint64_t v1, int tid) {
     constexpr int U = LC_COPY_UNROLL;
-    uint64_t v = v0 + threadIdx.x;
-    for (; v + (U - 1) * BS < v1; v += U * BS) {
+    uint64_t v = v0 + tid;
+    for (; v + (U - 1) * NT < v1; v += U * NT) {
         uint4 x[U];
 #pragma unroll
-        for (int u = 0; u < U; ++u) x[u] = ld_nc(src + 16 * (v + uint64_t(u) * BS));
+        for (int u = 0; u < U; ++u) x[u] = ld_nc(src + 16 * (v + uint64_t(u) * NT));
 #pragma unroll
-        for (int u = 0; u < U; ++u) st_v4(dst + 16 * (v + uint64_t(u) * BS), x[u]);
+        for (int u = 0; u < U; ++u) st_v4(dst + 16 * (v + uint64_t(u) * NT), x[u]);
         if (dst2) {
 #pragma unroll
-            for (int u = 0; u < U; ++u) st_v4(dst2 + 16 * (v + uint64_t(u) * BS), x[u]);
+            for (int u = 0; u < U; ++u) st_v4(dst2 + 16 * (v + uint64_t(u) * NT), x[u]);
         }
     }
-    for (; v < v1; v += BS) {
+    for (; v < v1; v += NT) {
         const uint4 x = ld_nc(src + 16 * v);
         st_v4(dst + 16 * v, x);
         if (dst2) st_v4(dst2 + 16 * v, x);
@@ -80,92 +84,348 @@ __device__ __forceinline__ void copy_vec(const uint8_t* src, uint8_t* dst, uint8
 }
 
 // Units of T (4, 2 or 1 bytes) [u0, u1) of an entry.
-template <typename T>
+template <typename T, int NT>
 __device__ __forceinline__ void copy_units(const uint8_t* src, uint8_t* dst, uint8_t* dst2,
-                                           uint64_t u0, uint64_t u1) {
+                                           uint64_t u0, uint64_t u1, int tid) {
     const T* s = reinterpret_cast<const T*>(src);
     T* d = reinterpret_cast<T*>(dst);
     T* d2 = reinterpret_cast<T*>(dst2);
-    for (uint64_t u = u0 + threadIdx.x; u < u1; u += BS) {
+    for (uint64_t u = u0 + tid; u < u1; u += NT) {
         const T x = s[u];
         d[u] = x;
         if (d2) d2[u] = x;
     }
 }
 
-__device__ __forceinline__ void zero_vec(uint8_t* dst, uint64_t v0, uint64_t v1) {
+template <int NT>
+__device__ __forceinline__ void zero_vec(uint8_t* dst, uint64_t v0, uint64_t v1, int tid) {
     const uint4 z = make_uint4(0u, 0u, 0u, 0u);
-    for (uint64_t v = v0 + threadIdx.x; v < v1; v += BS) st_v4(dst + 16 * v, z);
+    for (uint64_t v = v0 + tid; v < v1; v += NT) st_v4(dst + 16 * v, z);
 }
 
-// Bytes [a, b) of one entry, a and b multiples of 16 within [0, span].
-__device__ void copy_entry(const CopyParams& p, const CopyDesc& d, uint64_t a, uint64_t b) {
-    const uint8_t* src = p.mode == kScatter ? p.base + (d.woff - p.lo) : d.src;
-    uint8_t* dst = p.mode == kGather ? p.base + (d.woff - p.lo) : d.dst;
-    uint8_t* dst2 = d.dst2;
+// Resolved addresses of one entry for the launch's mode.
+struct EntryAddr {
+    const uint8_t* src;
+    uint8_t* dst;
+    uint8_t* dst2;
+    bool vec;   // src, dst and dst2 all 16-byte aligned
+};
+
+__device__ __forceinline__ EntryAddr entry_addr(const CopyParams& p, const CopyDesc& d) {
+    EntryAddr e;
+    e.src = p.mode == kScatter ? p.base + (d.woff - p.lo) : d.src;
+    e.dst = p.mode == kGather ? p.base + (d.woff - p.lo) : d.dst;
+    e.dst2 = d.dst2;
+    e.vec = ((uintptr_t(e.src) | uintptr_t(e.dst) | uintptr_t(e.dst2)) & 15) == 0;
+    return e;
+}
+
+// Bytes [a, b) of one entry, a and b multiples of 16 within [0, span], by
+// thread tid of NT workers.  With kBulkPayload the 16-byte vectors of the
+// payload of a vector-aligned entry are left to the bulk engine
+// (bulk_next_chunk takes exactly those); everything else -- sub-vector
+// tails, entries with misaligned addresses and the GATHER padding -- is
+// written here.
+template <int NT, bool kBulkPayload>
+__device__ void copy_entry(const CopyParams& p, const CopyDesc& d, uint64_t a, uint64_t b, int tid) {
+    const EntryAddr e = entry_addr(p, d);
     const uint64_t pe = b < d.nbytes ? b : d.nbytes;   // payload end inside [a, b)
     if (a < pe) {
-        const uintptr_t al = uintptr_t(src) | uintptr_t(dst) | uintptr_t(dst2);
+        const uintptr_t al = uintptr_t(e.src) | uintptr_t(e.dst) | uintptr_t(e.dst2);
         uint64_t done;   // payload bytes [a, done) handled by the unit loop
-        if ((al & 15) == 0) {
+        if (e.vec) {
             done = pe & ~uint64_t(15);
-            if (a < done) copy_vec(src, dst, dst2, a >> 4, done >> 4);
+            if (!kBulkPayload && a < done) copy_vec<NT>(e.src, e.dst, e.dst2, a >> 4, done >> 4, tid);
         } else if ((al & 3) == 0) {
             done = pe & ~uint64_t(3);
-            if (a < done) copy_units<uint32_t>(src, dst, dst2, a >> 2, done >> 2);
+            if (a < done) copy_units<uint32_t, NT>(e.src, e.dst, e.dst2, a >> 2, done >> 2, tid);
         } else if ((al & 1) == 0) {
             done = pe & ~uint64_t(1);
-            if (a < done) copy_units<uint16_t>(src, dst, dst2, a >> 1, done >> 1);
+            if (a < done) copy_units<uint16_t, NT>(e.src, e.dst, e.dst2, a >> 1, done >> 1, tid);
         } else {
             done = pe;
-            copy_units<uint8_t>(src, dst, dst2, a, pe);
+            copy_units<uint8_t, NT>(e.src, e.dst, e.dst2, a, pe, tid);
         }
-        if (threadIdx.x == 0) {
+        if (tid == 0) {
             for (uint64_t q = done > a ? done : a; q < pe; ++q) {
-                dst[q] = src[q];
-                if (dst2) dst2[q] = src[q];
+                e.dst[q] = e.src[q];
+                if (e.dst2) e.dst2[q] = e.src[q];
             }
         }
     }
     if (p.mode == kGather && b > d.nbytes) {
         const uint64_t z0 = a > d.nbytes ? a : d.nbytes;
         const uint64_t zv = (z0 + 15) & ~uint64_t(15);
-        if (threadIdx.x == 0)
-            for (uint64_t q = z0; q < zv && q < b; ++q) dst[q] = 0;
-        if (zv < b) zero_vec(dst, zv >> 4, b >> 4);
+        if (tid == 0)
+            for (uint64_t q = z0; q < zv && q < b; ++q) e.dst[q] = 0;
+        if (zv < b) zero_vec<NT>(e.dst, zv >> 4, b >> 4, tid);
     }
 }
 
-__global__ void __launch_bounds__(kCopyThreads) copy_kernel(CopyParams p) {
+// The CTA's work range [x, xe) (granules of LC_COPY_ALIGN_BYTES, the last
+// one ragged) and the last entry with woff <= x.  Returns false when the
+// CTA has nothing to do.
+__device__ __forceinline__ bool cta_range(CopyParams& p, uint64_t& x, uint64_t& xe, int& first) {
     if (p.ndesc_dev) {           // sizes decided on the device by the select kernel
         p.ndesc = *p.ndesc_dev;
         p.hi = p.lo + *p.hi_dev;
     }
-    // CTA ranges in granules of LC_COPY_ALIGN_BYTES (the last one ragged)
     constexpr uint64_t kGran = LC_COPY_ALIGN_BYTES / 16;
     const uint64_t units = (p.hi - p.lo) >> 4;
     const uint64_t grans = (units + kGran - 1) / kGran;
-    uint64_t u0 = grans * blockIdx.x / gridDim.x * kGran;
+    const uint64_t u0 = grans * blockIdx.x / gridDim.x * kGran;
     uint64_t u1 = grans * (blockIdx.x + 1) / gridDim.x * kGran;
     if (u1 > units) u1 = units;
-    if (u0 >= u1 || p.ndesc <= 0) return;
-    uint64_t x = p.lo + (u0 << 4);
-    const uint64_t xe = p.lo + (u1 << 4);
-    // last entry with woff <= x
+    if (u0 >= u1 || p.ndesc <= 0) return false;
+    x = p.lo + (u0 << 4);
+    xe = p.lo + (u1 << 4);
     int lo_i = 0, hi_i = p.ndesc - 1;
     while (lo_i < hi_i) {
         const int mid = (lo_i + hi_i + 1) >> 1;
         if (p.desc[mid].woff <= x) lo_i = mid;
         else hi_i = mid - 1;
     }
-    for (int i = lo_i; x < xe && i < p.ndesc; ++i) {
+    first = lo_i;
+    return true;
+}
+
+// Every entry overlapping [x, xe), clipped to it, through copy_entry.
+template <int NT, bool kBulkPayload>
+__device__ __forceinline__ void walk_entries(const CopyParams& p, int i, uint64_t x, uint64_t xe, int tid) {
+    for (; x < xe && i < p.ndesc; ++i) {
         const CopyDesc d = p.desc[i];
         const uint64_t ent_end = d.woff + d.span;
         if (ent_end <= x) continue;
         const uint64_t end = xe < ent_end ? xe : ent_end;
-        copy_entry(p, d, x - d.woff, end - d.woff);
+        copy_entry<NT, kBulkPayload>(p, d, x - d.woff, end - d.woff, tid);
         x = end;
     }
+}
+
+__global__ void __launch_bounds__(kCopyThreads) copy_kernel(CopyParams p) {
+    uint64_t x, xe;
+    int first;
+    if (!cta_range(p, x, xe, first)) return;
+    walk_entries<BS, false>(p, first, x, xe, threadIdx.x);
+}
+
+// ---------------------------------------------------------------------------
+// Bulk engine.  One thread of the CTA streams the 16-byte-aligned payload
+// through a ring of kStages shared-memory buffers: cp.async.bulk loads
+// global -> shared completing on one mbarrier per buffer, then
+// cp.async.bulk stores shared -> global (to dst and, for the fused commit,
+// dst2), tracked as bulk groups.  A buffer is refilled once the store that
+// read it has finished reading (wait_group.read), so kStages - 1 loads are
+// in flight behind the store being issued.  Warps 1.. walk the same range
+// for the rest (tails, misaligned entries, padding) with ordinary loads and
+// stores; the two sides write disjoint bytes and never synchronise.
+// ---------------------------------------------------------------------------
+#ifndef LC_BULK_STAGES
+#define LC_BULK_STAGES 6
+#endif
+#ifndef LC_BULK_CHUNK
+#define LC_BULK_CHUNK 32768
+#endif
+constexpr int kStages = LC_BULK_STAGES;
+constexpr uint32_t kChunk = LC_BULK_CHUNK;
+constexpr int kWorkers = BS - 32;
+constexpr size_t kBulkSmem = size_t(kStages) * kChunk;
+static_assert(kChunk % 16 == 0 && kStages >= 2, "bulk ring shape");
+// A wait gives up after this long (a 32 KB load completes in microseconds);
+// the iteration cap bounds it even if the timer were not advancing.
+constexpr uint64_t kWaitNs = 1000000000ull;
+constexpr uint64_t kDrainNs = 100000000ull;
+constexpr uint32_t kWaitIters = 1u << 28;
+
+struct BulkJob {
+    const uint8_t* src;
+    uint8_t* dst;
+    uint8_t* dst2;
+    uint32_t bytes;
+};
+
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t done;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return done != 0;
+}
+
+// Waits for the phase with the given parity to complete, for at most
+// `limit_ns` (and kWaitIters polls).  Returns false if it gave up.
+__device__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_ns();
+    for (uint32_t it = 0; it < kWaitIters; ++it) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (global_ns() - t0 > limit_ns) return false;
+    }
+    return false;
+}
+
+// Every byte is read once and written once: with LC_BULK_L2_HINT the
+// copies ask L2 to evict their lines first, so that the stream does not
+// push the next step's working set out (the thread kernel's .cs stores).
+#ifndef LC_BULK_L2_HINT
+#define LC_BULK_L2_HINT 1
+#endif
+
+__device__ __forceinline__ uint64_t evict_first_policy() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+
+__device__ __forceinline__ void bulk_load(uint32_t dst_smem, const void* src, uint32_t bytes, uint32_t bar,
+                                          uint32_t announced, uint64_t pol) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(announced) : "memory");
+#if LC_BULK_L2_HINT
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;"
+        ::"r"(dst_smem), "l"(src), "r"(bytes), "r"(bar), "l"(pol)
+        : "memory");
+#else
+    (void)pol;
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst_smem),
+        "l"(src), "r"(bytes), "r"(bar)
+        : "memory");
+#endif
+}
+
+__device__ __forceinline__ void bulk_store(void* dst, uint32_t src_smem, uint32_t bytes, uint64_t pol) {
+#if LC_BULK_L2_HINT
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group.L2::cache_hint [%0], [%1], %2, %3;" ::"l"(dst),
+                 "r"(src_smem), "r"(bytes), "l"(pol)
+                 : "memory");
+#else
+    (void)pol;
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst), "r"(src_smem),
+                 "r"(bytes)
+                 : "memory");
+#endif
+}
+
+// Next chunk (at most kChunk bytes) of 16-byte-aligned payload at or after
+// work position x, advancing x (and the entry index i) past it.  Takes
+// exactly the bytes copy_entry<..., true> leaves out.
+__device__ bool bulk_next_chunk(const CopyParams& p, int& i, uint64_t& x, uint64_t xe, BulkJob& j) {
+    while (x < xe && i < p.ndesc) {
+        const CopyDesc d = p.desc[i];
+        const uint64_t ent_end = d.woff + d.span;
+        if (ent_end <= x) {
+            ++i;
+            continue;
+        }
+        const uint64_t end = xe < ent_end ? xe : ent_end;
+        const uint64_t a = x - d.woff, b = end - d.woff;
+        const EntryAddr e = entry_addr(p, d);
+        const uint64_t pv = (b < d.nbytes ? b : d.nbytes) & ~uint64_t(15);
+        if (e.vec && a < pv) {
+            const uint64_t n = pv - a < kChunk ? pv - a : kChunk;
+            j.src = e.src + a;
+            j.dst = e.dst + a;
+            j.dst2 = e.dst2 ? e.dst2 + a : nullptr;
+            j.bytes = uint32_t(n);
+            x += n;
+            return true;
+        }
+        x = end;
+        ++i;
+    }
+    return false;
+}
+
+__device__ void bulk_drive(const CopyParams& p, int i, uint64_t x, uint64_t xe, uint8_t* ring, uint64_t* bars,
+                           BulkJob* jobs) {
+    const uint32_t ring_s = smem_addr(ring);
+    const uint32_t bar_s = smem_addr(bars);
+    for (int s = 0; s < kStages; ++s) mbar_init(bar_s + 8 * s);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    const uint64_t pol = evict_first_policy();
+    uint32_t parity = 0;   // bit s: parity of the next phase of buffer s
+    uint64_t issued = 0, retired = 0;
+    bool more = true;
+    auto issue = [&]() {
+        BulkJob j;
+        if (!bulk_next_chunk(p, i, x, xe, j)) {
+            more = false;
+            return;
+        }
+        const int s = int(issued % kStages);
+        jobs[s] = j;
+        const uint32_t announced = j.bytes + (p.stall_first && issued == 0 ? 16u : 0u);
+        bulk_load(ring_s + uint32_t(s) * kChunk, j.src, j.bytes, bar_s + 8 * s, announced, pol);
+        ++issued;
+    };
+    while (more && issued < kStages - 1) issue();
+    bool ok = true;
+    while (retired < issued) {
+        const int s = int(retired % kStages);
+        if (!mbar_wait_bounded(bar_s + 8 * s, (parity >> s) & 1u, kWaitNs)) {
+            ok = false;
+            break;
+        }
+        parity ^= 1u << s;
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        const BulkJob j = jobs[s];
+        bulk_store(j.dst, ring_s + uint32_t(s) * kChunk, j.bytes, pol);
+        if (j.dst2) bulk_store(j.dst2, ring_s + uint32_t(s) * kChunk, j.bytes, pol);
+        asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+        ++retired;
+        if (more) {
+            // the buffer of chunk retired-2 is refilled: its store group,
+            // all but the newest, must have finished reading it
+            asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+            issue();
+        }
+    }
+    if (!ok) {
+        if (p.fault) {
+            *reinterpret_cast<volatile uint32_t*>(p.fault) = 1u;
+            __threadfence_system();
+        }
+        // let the loads still in flight land before the CTA's shared memory goes away
+        for (; retired < issued; ++retired) {
+            const int s = int(retired % kStages);
+            mbar_wait_bounded(bar_s + 8 * s, (parity >> s) & 1u, kDrainNs);
+            parity ^= 1u << s;
+        }
+    }
+    asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+
+__global__ void __launch_bounds__(kCopyThreads, 1) copy_bulk_kernel(CopyParams p) {
+    extern __shared__ __align__(128) uint8_t ring[];
+    __shared__ __align__(8) uint64_t bars[kStages];
+    __shared__ BulkJob jobs[kStages];
+    uint64_t x, xe;
+    int first;
+    if (!cta_range(p, x, xe, first)) return;
+    if (threadIdx.x < 32) {
+        if (threadIdx.x == 0) bulk_drive(p, first, x, xe, ring, bars, jobs);
+        return;
+    }
+    walk_entries<kWorkers, true>(p, first, x, xe, int(threadIdx.x) - 32);
 }
 
 }  // namespace
@@ -178,6 +438,20 @@ cudaError_t launch_copy(const CopyParams& p, int grid, cudaStream_t s) {
 
 cudaError_t copy_occupancy(int* blocks_per_sm) {
     return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, copy_kernel, kCopyThreads, 0);
+}
+
+cudaError_t launch_copy_bulk(const CopyParams& p, int grid, cudaStream_t s) {
+    cudaGetLastError();
+    copy_bulk_kernel<<<grid, kCopyThreads, kBulkSmem, s>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t copy_bulk_prepare(int* blocks_per_sm) {
+    cudaError_t e = cudaFuncSetAttribute(copy_bulk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         int(kBulkSmem));
+    if (e != cudaSuccess) return e;
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, copy_bulk_kernel, kCopyThreads,
+                                                         kBulkSmem);
 }
 
 }  // namespace lc

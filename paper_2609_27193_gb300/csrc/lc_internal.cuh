@@ -83,6 +83,12 @@ struct CopyParams {
     // and the end of the range are read from device memory at kernel start.
     const int32_t* ndesc_dev;
     const uint64_t* hi_dev;
+    // Host-mapped word a bulk-engine copy sets to 1 when a bounded wait
+    // runs out (never cleared by the device).
+    uint32_t* fault;
+    // Test of that bound: each CTA's first bulk load announces 16 bytes more
+    // than it brings, so its wait can only run out.
+    int32_t stall_first;
 };
 
 // A section of a layer's packed block (one segment's W, exp_avg or exp_avg_sq).
@@ -183,6 +189,11 @@ cudaError_t launch_adamw_measure(const MeasureParams& p, const OptSegDev* opt, c
 cudaError_t launch_select(const SelectParams& p, cudaStream_t s);
 cudaError_t launch_copy(const CopyParams& p, int grid, cudaStream_t s);
 cudaError_t copy_occupancy(int* blocks_per_sm);
+// Bulk-engine copy (cp.async.bulk through shared memory); every address the
+// launch touches must be device memory.  copy_bulk_prepare raises the
+// kernel's shared-memory limit and reports its CTAs per SM.
+cudaError_t launch_copy_bulk(const CopyParams& p, int grid, cudaStream_t s);
+cudaError_t copy_bulk_prepare(int* blocks_per_sm);
 
 // Sets the thread-local message returned by lc_last_error().
 void set_last_error(const char* msg);

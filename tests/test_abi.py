@@ -17,7 +17,7 @@ HEADER = os.path.join(ROOT, "include", "layercheck.h")
 def declared_functions():
     text = open(HEADER).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return set(re.findall(r"\b(lc_[a-z_]+)\s*\(", text))
+    return set(re.findall(r"\b(lc_[a-z0-9_]+)\s*\(", text))
 
 
 @pytest.fixture(scope="module")
@@ -54,7 +54,7 @@ def test_struct_layout_matches_c(lib):
     from paper_2609_27193_gb300 import _abi
     structs = {"lc_segment": _abi.lc_segment, "lc_config": _abi.lc_config,
                "lc_select_info": _abi.lc_select_info, "lc_version": _abi.lc_version,
-               "lc_counters": _abi.lc_counters}
+               "lc_counters": _abi.lc_counters, "lc_manifest_record": _abi.lc_manifest_record}
     lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "layercheck.h"',
              "int main(void) {"]
     for name, cls in structs.items():

@@ -27,9 +27,10 @@ def _assert_device_equals(st, comp, what="composite"):
             assert np.array_equal(st.host("v", k), v), "%s v of tensor %d" % (what, k)
 
 
+@pytest.mark.parametrize("engine", ["threads", "bulk"])
 @pytest.mark.parametrize("align", [16, 256, 4096])
 @pytest.mark.parametrize("alloc", ["separate", "flat", "skew"])
-def test_pack_device_bytes_and_fused_commit(align, alloc):
+def test_pack_device_bytes_and_fused_commit(align, alloc, engine):
     torch = require_gpu()
     sizes = [(n, i % 3) for i, n in enumerate([1, 7, 4096, 9, 100003, 33, 2, 65536, 5])]
     spec = custom_shape(sizes)
@@ -38,7 +39,7 @@ def test_pack_device_bytes_and_fused_commit(align, alloc):
     st = gen.SyntheticState(spec, device="cuda", seed=4, alloc=alloc, dtypes=dts,
                             moments_mask=moments)
     st.drift(1, np.array([1e-2, 1e-5, 1e-2]))
-    lc = make_lc(st, pack_align=align)
+    lc = make_lc(st, pack_align=align, copy_engine=engine)
     run = make_oracle(st, align=align)
     lc.measure(1)
     mask, u, nbytes = lc.select(1e-3, 100)
@@ -61,6 +62,9 @@ def test_pack_device_bytes_and_fused_commit(align, alloc):
     run.commit(run.last_mask, W)
     for k in range(len(sizes)):
         assert np.array_equal(st.host("R", k), run.R[k]), "snapshot of tensor %d" % k
+    c = lc.counters()
+    assert c["copy_launches"] == 1
+    assert c["bulk_copy_launches"] == (1 if engine == "bulk" else 0)
     lc.close()
 
 
@@ -90,8 +94,9 @@ def test_commit_unfused_and_accumulate_mode():
         lc.close()
 
 
+@pytest.mark.parametrize("engine", ["threads", "bulk"])
 @pytest.mark.parametrize("per_layer", [0, 2])
-def test_pack_async_store_and_restore_tiny(per_layer):
+def test_pack_async_store_and_restore_tiny(per_layer, engine):
     """The tiny workload for 20 steps (tau 1e-3, S_max 4), every step through
     the pinned store with a small staging ring (many chunks); masks, u and
     every persisted block against the oracle; then restores at several
@@ -103,7 +108,7 @@ def test_pack_async_store_and_restore_tiny(per_layer):
     spec = wl.shape()
     st = gen.SyntheticState(spec, device="cuda", seed=wl.seed)
     scales = wl.layer_scales(spec)
-    lc = make_lc(st, staging_bytes=2 << 20)
+    lc = make_lc(st, staging_bytes=2 << 20, copy_engine=engine)
     run = make_oracle(st)
     full = sum(lc.layer_block_bytes(l) for l in range(spec.nlayers))
     store = P.Store(lc, capacity_bytes=(wl.steps + 2) * full, versions_per_layer=per_layer)
@@ -158,6 +163,8 @@ def test_pack_async_store_and_restore_tiny(per_layer):
         assert steps.tolist() == [run.versions[p]["step"] for p in pick]
         torch.cuda.synchronize()
         _assert_device_equals(st, comp, "restore@%d" % t_fail)
+    c = lc.counters()
+    assert c["bulk_copy_launches"] == (c["copy_launches"] if engine == "bulk" else 0)
     store.close()
     lc.close()
 
@@ -238,12 +245,13 @@ def test_store_capacity_and_layout_checks():
 
 def test_pack_into_pinned_host_memory_directly():
     """lc_pack_device also accepts pinned host memory: the gather writes the
-    packed stream straight into it over the host link."""
+    packed stream straight into it over the host link (on the thread
+    engine, even when the bulk engine is asked for)."""
     torch = require_gpu()
     spec = shapes.tiny()
     st = gen.SyntheticState(spec, device="cuda", seed=3)
     st.drift(1, np.full(spec.nlayers, 1e-2))
-    lc = make_lc(st)
+    lc = make_lc(st, copy_engine="bulk")
     run = make_oracle(st)
     lc.measure(1)
     mask, u, nbytes = lc.select(1e-3, 100)
@@ -257,4 +265,99 @@ def test_pack_into_pinned_host_memory_directly():
     lc.commit_snapshot()
     torch.cuda.synchronize()
     assert np.array_equal(host.numpy(), stream)
+    # host memory is never handed to the bulk engine
+    assert lc.counters()["bulk_copy_launches"] == 0
     lc.close()
+
+
+@pytest.mark.parametrize("alloc", ["separate", "skew"])
+def test_bulk_engine_long_ranges(alloc):
+    """The tiny workload packed whole with both engines: every CTA streams
+    many 32 KB chunks through its ring and entries straddle CTA ranges;
+    "skew" puts every snapshot one element off 16-byte alignment, so the W
+    sections (whose fused commit writes the snapshot) take the thread path
+    inside the bulk kernel while the moments take the bulk path.  Streams
+    and snapshots against the oracle, and the two engines against each
+    other."""
+    torch = require_gpu()
+    spec = shapes.tiny()
+    out = {}
+    for engine in ("bulk", "threads"):
+        st = gen.SyntheticState(spec, device="cuda", seed=12, alloc=alloc)
+        st.drift(1, np.full(spec.nlayers, 1e-2))
+        lc = make_lc(st, copy_engine=engine)
+        run = make_oracle(st)
+        lc.measure(1)
+        mask, u, nbytes = lc.select(1e-3, 100)
+        W, M, V = _host(st)
+        ou, _ = run.measure(W)
+        run.select(ou, 1e-3, 100, 1)
+        compare_decision(mask, u, run, ou, 1e-3)
+        assert mask.all()
+        stream, _ = run.pack(run.last_mask, W, M, V, 1)
+        dst = torch.full((nbytes + 512,), 0x5A, dtype=torch.uint8, device="cuda")
+        lc.pack_device(dst)
+        lc.commit_snapshot()
+        torch.cuda.synchronize()
+        got = dst.cpu().numpy()
+        assert np.array_equal(got[:nbytes], stream), engine
+        assert np.all(got[nbytes:] == 0x5A), engine
+        run.commit(run.last_mask, W)
+        for k in range(len(spec.tensors)):
+            assert np.array_equal(st.host("R", k), run.R[k]), (engine, k)
+        c = lc.counters()
+        assert c["bulk_copy_launches"] == (1 if engine == "bulk" else 0)
+        out[engine] = got[:nbytes]
+        lc.close()
+    assert np.array_equal(out["bulk"], out["threads"])
+
+
+def test_bulk_engine_wait_bound_reports_timeout():
+    """LC_DEBUG_BULK_STALL makes each CTA of a bulk copy wait for 16 bytes
+    that never arrive.  The bounded wait runs out (1 s), the launch returns,
+    and the host reads the context's copy-fault word: lc_wait_durable and
+    every later lc_select fail with LC_ERR_TIMEOUT.  The CUDA context stays
+    usable: a fresh library context on the same state packs correctly."""
+    import time
+    torch = require_gpu()
+    import paper_2609_27193_gb300 as P
+    spec = shapes.tiny()
+    st = gen.SyntheticState(spec, device="cuda", seed=2)
+    st.drift(1, np.full(spec.nlayers, 1e-2))
+    lc = make_lc(st, copy_engine="bulk", debug_flags=P.LC_DEBUG_BULK_STALL)
+    store = P.Store(lc, versions_per_layer=2)
+    lc.measure(1)
+    mask, u, nbytes = lc.select(1e-3, 100)
+    assert nbytes > 0
+    t0 = time.perf_counter()
+    lc.pack_async(store)
+    lc.commit_snapshot()
+    with pytest.raises(P.LCError) as e:
+        lc.wait_durable(1)
+    assert e.value.status == 6
+    assert time.perf_counter() - t0 < 30.0
+    assert lc.counters()["bulk_copy_launches"] == 1
+    lc.measure(2)
+    with pytest.raises(P.LCError) as e:
+        lc.select(1e-3, 100)
+    assert e.value.status == 6
+    store.close()
+    lc.close()
+    x = torch.arange(1 << 20, device="cuda", dtype=torch.float64)
+    assert float(x.sum()) == float((1 << 20) * ((1 << 20) - 1) // 2)
+    st2 = gen.SyntheticState(spec, device="cuda", seed=2)
+    st2.drift(1, np.full(spec.nlayers, 1e-2))
+    lc2 = make_lc(st2, copy_engine="bulk")
+    run = make_oracle(st2)
+    lc2.measure(1)
+    mask, u, nbytes = lc2.select(1e-3, 100)
+    W, M, V = _host(st2)
+    ou, _ = run.measure(W)
+    run.select(ou, 1e-3, 100, 1)
+    stream, _ = run.pack(run.last_mask, W, M, V, 1)
+    dst = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    lc2.pack_device(dst)
+    torch.cuda.synchronize()
+    assert np.array_equal(dst.cpu().numpy(), stream)
+    assert lc2.counters()["bulk_copy_launches"] == 1
+    lc2.close()
