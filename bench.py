@@ -57,9 +57,9 @@ def parse_args():
                     help="scan: measure against the snapshot (default); fused: AdamW step with "
                          "the drift read off the update, fp32 master weights; graph: the scan "
                          "step replayed as one captured CUDA graph with no host round trip")
-    ap.add_argument("--copy-engine", choices=["threads", "bulk"], default="threads",
-                    help="threads: per-thread 16-byte vector copies (default); bulk: the "
-                         "bulk-copy engine through shared memory when every buffer is device memory")
+    ap.add_argument("--copy-engine", choices=["bulk", "threads"], default="bulk",
+                    help="bulk: the bulk-copy engine through shared memory when every buffer is "
+                         "device memory (default); threads: per-thread 16-byte vector copies")
     ap.add_argument("--lean", action="store_true",
                     help="no fp32 master weights in the generator (small case for kernel captures)")
     return ap.parse_args()
@@ -97,7 +97,7 @@ def kernel_source_sha(files):
 KERNEL_FILES = {"measure": ["lc_measure.cu", "lc_reduce.cuh", "lc_internal.cuh"],
                 "fused_adamw": ["lc_adamw.cu", "lc_reduce.cuh", "lc_internal.cuh"],
                 "pack": ["lc_copy.cu", "lc_internal.cuh"],
-                "pack_bulk": ["lc_copy.cu", "lc_internal.cuh"]}
+                "pack_threads": ["lc_copy.cu", "lc_internal.cuh"]}
 
 
 def profiled_traffic(kernel, workload, persisted_bytes=None):
@@ -327,18 +327,6 @@ def reference_arm(args):
 # our arm
 # ---------------------------------------------------------------------------
 
-def first_blocks(shape, nblocks):
-    """The first `nblocks` transformer blocks of a shape, layers renumbered."""
-    from lc_workloads.shapes import ModelShape, TensorSpec
-    blocks = [l for l in range(shape.nlayers) if shape.layer_names[l].startswith("block")]
-    keep = blocks[:nblocks] if blocks else list(range(min(nblocks, shape.nlayers)))
-    ts = [TensorSpec(t.name, keep.index(t.layer), t.numel, t.dtype)
-          for t in shape.tensors if t.layer in keep]
-    sub = ModelShape("%s-first%d" % (shape.name, len(keep)), 0, 0, 0, 0, 0, 0, 0, False, False,
-                     ts, len(keep), [shape.layer_names[l] for l in keep])
-    return sub, keep
-
-
 def d2h_link_probe(torch, dev, nbytes=4 << 30):
     """Plain device->pinned-host copy bandwidth measured beside the e2e loop
     (the host link is shared with other jobs on the machine, so it varies)."""
@@ -377,13 +365,14 @@ def run_ours(args):
     dev = torch.device("cuda", local)
     P = load_package()
     from lc_workloads import gen
+    from lc_workloads import shapes
     from lc_workloads.configs import WORKLOADS, cadence_scales
 
     wl = WORKLOADS[args.workload]
     shape = wl.shape()
     base_scales = wl.layer_scales(shape)
     if args.shape_blocks > 0:
-        shape, keep = first_blocks(shape, args.shape_blocks)
+        shape, keep = shapes.first_blocks(shape, args.shape_blocks)
         base_scales = base_scales[keep]
     tau = float(args.tau if args.tau is not None else wl.tau)
     K = wl.max_staleness
@@ -560,7 +549,7 @@ def run_ours(args):
     dominant = "measure" if sum(measure_ms) >= sum(pack_ms) else "pack"
     measure_name = "fused_adamw" if fused else "measure"
     mean_persisted = statistics.mean(r["nbytes"] for r in recs)
-    pack_name = "pack" if args.copy_engine == "threads" else "pack_bulk"
+    pack_name = "pack" if args.copy_engine == "bulk" else "pack_threads"
     traffic, tsrc = profiled_traffic(measure_name if dominant == "measure" else pack_name,
                                      args.workload, mean_persisted if dominant == "pack" else None)
     if fused and dominant == "pack":
@@ -605,11 +594,13 @@ def run_ours(args):
         except OSError:
             pass
         cap = full if avail == 0 else min(full, int(avail * 0.6))
+        # the pinned destination holds one step (the log store is cleared
+        # after every step): room for twice the largest step of the device loop
+        cap = min(cap, int(max(r["nbytes"] for r in recs) * 2) + (64 << 20))
         if graph:
             # the replayed pack writes straight into pinned host memory
             store = None
-            hcap = min(cap, int(max(r["nbytes"] for r in recs) * 1.5) + (64 << 20))
-            hostdst = torch.empty(hcap, dtype=torch.uint8, pin_memory=True)
+            hostdst = torch.empty(cap, dtype=torch.uint8, pin_memory=True)
             lc.step_graph_create(tau, K, hostdst)
         else:
             store = P.Store(lc, capacity_bytes=cap)

@@ -73,13 +73,13 @@ typedef enum { LC_DRIFT_SNAPSHOT = 0, LC_DRIFT_ACCUMULATE = 1 } lc_drift_mode;
 
 /* Kernel that moves packed, committed and restored bytes (the bytes are the
  * same either way).
- * LC_COPY_THREADS: every thread loads and stores 16-byte vectors (default;
- *                  the faster one on the packs measured so far).
  * LC_COPY_BULK   : the bulk-copy engine (cp.async.bulk through shared
- *                  memory) whenever every address of the copy is device
- *                  memory -- segments, staging ring and destination -- else
- *                  as LC_COPY_THREADS. */
-typedef enum { LC_COPY_THREADS = 0, LC_COPY_BULK = 1 } lc_copy_engine;
+ *                  memory, one load-issuing and one store-issuing thread per
+ *                  SM) whenever every address of the copy is device memory
+ *                  -- segments, staging ring and destination -- else as
+ *                  LC_COPY_THREADS (default).
+ * LC_COPY_THREADS: every thread loads and stores 16-byte vectors. */
+typedef enum { LC_COPY_BULK = 0, LC_COPY_THREADS = 1 } lc_copy_engine;
 
 /* LC_DEBUG_BULK_STALL: every bulk-engine copy launch waits for 16 bytes that
  * never arrive, once per CTA.  The engine's bounded wait (1 s) runs out, the
@@ -125,7 +125,7 @@ typedef struct {
     int32_t timeout_ms;      /* bound of every host wait (default 60000)          */
     uint64_t staging_bytes;  /* device staging ring used by lc_pack_async and
                                 lc_restore, split in two slots (default 512 MiB) */
-    int32_t copy_engine;     /* lc_copy_engine (default LC_COPY_THREADS)         */
+    int32_t copy_engine;     /* lc_copy_engine (default LC_COPY_BULK)            */
     int32_t debug_flags;     /* 0, or LC_DEBUG_BULK_STALL (tests only)           */
 } lc_config;
 

@@ -170,6 +170,15 @@ class SyntheticState:
                 if redraw_moments:
                     self._draw_moments(step, k)
 
+    def resync_master(self):
+        """After a recovery wrote W on the device: the fp32 master copy
+        restarts from the restored weights."""
+        if not self.master:
+            return
+        with torch.no_grad():
+            for k in range(len(self.specs)):
+                self.M[k].copy_(self.W[k])
+
     def set_values(self, k, w=None, r=None):
         """Overwrite W (and M) and/or R of tensor k with given float values."""
         with torch.no_grad():

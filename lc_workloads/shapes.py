@@ -89,3 +89,15 @@ def llama3_8b(per_tensor=False):
     vocab 128256, untied head (35 layers; 291 tensors)."""
     return decoder_shape("llama3-8b" + ("-per-tensor" if per_tensor else ""), 32, 4096, 14336,
                          32, 8, 128, 128256, tied=False, per_tensor=per_tensor)
+
+
+def first_blocks(shape, nblocks):
+    """The first `nblocks` transformer blocks of a shape as a shape of their
+    own (layers renumbered from 0), and the original layer ids kept."""
+    blocks = [l for l in range(shape.nlayers) if shape.layer_names[l].startswith("block")]
+    keep = blocks[:nblocks] if blocks else list(range(min(nblocks, shape.nlayers)))
+    ts = [TensorSpec(t.name, keep.index(t.layer), t.numel, t.dtype)
+          for t in shape.tensors if t.layer in keep]
+    sub = ModelShape("%s-first%d" % (shape.name, len(keep)), 0, 0, 0, 0, 0, 0, 0, False, False,
+                     ts, len(keep), [shape.layer_names[l] for l in keep])
+    return sub, keep

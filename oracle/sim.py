@@ -139,6 +139,30 @@ class OracleRun:
         stream = np.concatenate(parts) if parts else np.zeros(0, np.uint8)
         return stream, offsets
 
+    def record(self, mask, t):
+        """The versions a step persists, recorded without their bytes (the
+        pick of §3.5 needs only layer and step).  For long runs that check
+        the composite at chosen steps only: §3.3 keeps every layer's newest
+        version within the last S_max steps, so packing (pack) over the
+        S_max steps before a check is enough to hold every block it picks."""
+        off = 0
+        for l in range(self.nlayers):
+            if not mask[l]:
+                continue
+            nb = self._block_bytes(l)
+            self.versions.append(dict(layer=l, step=int(t), durable=False, digest=None,
+                                      nbytes=nb, offset=off))
+            if self.keep_blocks != "all":
+                for j in [j for j in self.blocks if self.versions[j]["layer"] == l]:
+                    del self.blocks[j]
+            off += nb
+
+    def _block_bytes(self, l):
+        cache = self.__dict__.setdefault("_block_bytes_cache", {})
+        if l not in cache:
+            cache[l] = int(self.layer_block_bytes(l))
+        return cache[l]
+
     def commit(self, mask, W):
         """Snapshot mode: R_l <- W_l(t) for the persisted layers (Eq. 4 resets
         the drift reference together with the accumulator)."""

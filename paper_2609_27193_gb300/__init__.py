@@ -85,14 +85,14 @@ class LayerCheck:
 
     def __init__(self, device=0, stream=None, eps_w=1e-8, mode=LC_DRIFT_SNAPSHOT,
                  pack_align=256, fuse_commit=True, timeout_ms=60000, staging_bytes=512 << 20,
-                 copy_engine="threads", debug_flags=0):
+                 copy_engine="bulk", debug_flags=0):
         lib = library()
         cfg = lc_config()
         lib.lc_config_default(C.byref(cfg))
         cfg.eps_w, cfg.mode, cfg.pack_align = float(eps_w), int(mode), int(pack_align)
         cfg.fuse_commit, cfg.timeout_ms = int(bool(fuse_commit)), int(timeout_ms)
         cfg.staging_bytes = int(staging_bytes)
-        engines = {"threads": LC_COPY_THREADS, "bulk": LC_COPY_BULK}
+        engines = {"bulk": LC_COPY_BULK, "threads": LC_COPY_THREADS}
         if copy_engine not in engines:
             raise ValueError("copy_engine must be one of %s" % sorted(engines))
         cfg.copy_engine = engines[copy_engine]

@@ -22,7 +22,7 @@ STATUS_NAMES = {0: "LC_OK", 1: "LC_ERR_INVALID_ARG", 2: "LC_ERR_STATE", 3: "LC_E
 
 LC_BF16, LC_F32 = 0, 1
 LC_DRIFT_SNAPSHOT, LC_DRIFT_ACCUMULATE = 0, 1
-LC_COPY_THREADS, LC_COPY_BULK = 0, 1
+LC_COPY_BULK, LC_COPY_THREADS = 0, 1
 LC_DEBUG_BULK_STALL = 1
 
 

@@ -1,8 +1,9 @@
 // lc_copy.cu -- the byte-moving kernels behind the pack (§3.1 full layer
 // state into one contiguous stream), the snapshot commit and the restore
-// scatter (§3.5): copy_kernel (every thread loads and stores 16-byte
-// vectors) and copy_bulk_kernel (the payload goes through shared memory on
-// the bulk-copy engine; used when every address is device memory).
+// scatter (§3.5): copy_bulk_kernel (the payload goes through shared memory
+// on the bulk-copy engine; the default whenever every address is device
+// memory) and copy_kernel (every thread loads and stores 16-byte vectors;
+// used for host memory and on request).
 //
 // A launch covers the work range [lo, hi) of a descriptor list whose
 // entries tile a linear work space (lc_internal.cuh).  The range is cut into
@@ -210,27 +211,34 @@ __global__ void __launch_bounds__(kCopyThreads) copy_kernel(CopyParams p) {
 }
 
 // ---------------------------------------------------------------------------
-// Bulk engine.  One thread of the CTA streams the 16-byte-aligned payload
-// through a ring of kStages shared-memory buffers: cp.async.bulk loads
-// global -> shared completing on one mbarrier per buffer, then
-// cp.async.bulk stores shared -> global (to dst and, for the fused commit,
-// dst2), tracked as bulk groups.  A buffer is refilled once the store that
-// read it has finished reading (wait_group.read), so kStages - 1 loads are
-// in flight behind the store being issued.  Warps 1.. walk the same range
-// for the rest (tails, misaligned entries, padding) with ordinary loads and
-// stores; the two sides write disjoint bytes and never synchronise.
+// Bulk engine.  The 16-byte-aligned payload streams through a ring of
+// kStages shared-memory buffers.  One thread (warp 0) is the producer: it
+// issues cp.async.bulk loads global -> shared, each completing on the
+// buffer's "full" mbarrier.  Another (warp 1) is the consumer: it waits for
+// a full buffer and issues cp.async.bulk stores shared -> global (dst and,
+// for the fused commit, dst2), one bulk group per buffer; once the group of
+// buffer k has finished reading shared memory (wait_group.read, kLag groups
+// behind) it arrives on that buffer's "empty" mbarrier, which the producer
+// waits for before it refills the buffer.  A job with zero bytes marks the
+// end of the CTA's range.  Warps 2.. walk the same range for the rest
+// (tails, misaligned entries, padding) with ordinary loads and stores; the
+// two sides write disjoint bytes and never synchronise.
 // ---------------------------------------------------------------------------
 #ifndef LC_BULK_STAGES
-#define LC_BULK_STAGES 6
+#define LC_BULK_STAGES 4
 #endif
 #ifndef LC_BULK_CHUNK
 #define LC_BULK_CHUNK 32768
 #endif
+#ifndef LC_BULK_LAG
+#define LC_BULK_LAG 2
+#endif
 constexpr int kStages = LC_BULK_STAGES;
 constexpr uint32_t kChunk = LC_BULK_CHUNK;
-constexpr int kWorkers = BS - 32;
+constexpr int kLag = LC_BULK_LAG;         // store groups still reading shared memory
+constexpr int kWorkers = BS - 64;
 constexpr size_t kBulkSmem = size_t(kStages) * kChunk;
-static_assert(kChunk % 16 == 0 && kStages >= 2, "bulk ring shape");
+static_assert(kChunk % 16 == 0 && kStages >= 2 && kLag >= 1 && kLag < kStages, "bulk ring shape");
 // A wait gives up after this long (a 32 KB load completes in microseconds);
 // the iteration cap bounds it even if the timer were not advancing.
 constexpr uint64_t kWaitNs = 1000000000ull;
@@ -282,12 +290,14 @@ __device__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, uint64_t limit_
     return false;
 }
 
-// Every byte is read once and written once: with LC_BULK_L2_HINT the
-// copies ask L2 to evict their lines first, so that the stream does not
-// push the next step's working set out (the thread kernel's .cs stores).
+// Every byte is read once and written once.  LC_BULK_L2_HINT asks L2 to
+// evict the copies' lines first: 0 never, 1 loads and stores, 2 loads only,
+// 3 stores only.
 #ifndef LC_BULK_L2_HINT
-#define LC_BULK_L2_HINT 1
+#define LC_BULK_L2_HINT 0
 #endif
+#define LC_BULK_HINT_LOADS (LC_BULK_L2_HINT == 1 || LC_BULK_L2_HINT == 2)
+#define LC_BULK_HINT_STORES (LC_BULK_L2_HINT == 1 || LC_BULK_L2_HINT == 3)
 
 __device__ __forceinline__ uint64_t evict_first_policy() {
     uint64_t pol;
@@ -298,7 +308,7 @@ __device__ __forceinline__ uint64_t evict_first_policy() {
 __device__ __forceinline__ void bulk_load(uint32_t dst_smem, const void* src, uint32_t bytes, uint32_t bar,
                                           uint32_t announced, uint64_t pol) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(announced) : "memory");
-#if LC_BULK_L2_HINT
+#if LC_BULK_HINT_LOADS
     asm volatile(
         "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;"
         ::"r"(dst_smem), "l"(src), "r"(bytes), "r"(bar), "l"(pol)
@@ -313,7 +323,7 @@ __device__ __forceinline__ void bulk_load(uint32_t dst_smem, const void* src, ui
 }
 
 __device__ __forceinline__ void bulk_store(void* dst, uint32_t src_smem, uint32_t bytes, uint64_t pol) {
-#if LC_BULK_L2_HINT
+#if LC_BULK_HINT_STORES
     asm volatile("cp.async.bulk.global.shared::cta.bulk_group.L2::cache_hint [%0], [%1], %2, %3;" ::"l"(dst),
                  "r"(src_smem), "r"(bytes), "l"(pol)
                  : "memory");
@@ -355,60 +365,73 @@ __device__ bool bulk_next_chunk(const CopyParams& p, int& i, uint64_t& x, uint64
     return false;
 }
 
-__device__ void bulk_drive(const CopyParams& p, int i, uint64_t x, uint64_t xe, uint8_t* ring, uint64_t* bars,
-                           BulkJob* jobs) {
-    const uint32_t ring_s = smem_addr(ring);
-    const uint32_t bar_s = smem_addr(bars);
-    for (int s = 0; s < kStages; ++s) mbar_init(bar_s + 8 * s);
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void bulk_fault(const CopyParams& p) {
+    if (p.fault) {
+        *reinterpret_cast<volatile uint32_t*>(p.fault) = 1u;
+        __threadfence_system();
+    }
+}
+
+struct BulkRing {
+    uint64_t full[kStages];
+    uint64_t empty[kStages];
+    BulkJob jobs[kStages];
+};
+
+__device__ void bulk_produce(const CopyParams& p, int i, uint64_t x, uint64_t xe, uint32_t ring_s, BulkRing& r) {
+    const uint32_t full_s = smem_addr(r.full), empty_s = smem_addr(r.empty);
     const uint64_t pol = evict_first_policy();
-    uint32_t parity = 0;   // bit s: parity of the next phase of buffer s
-    uint64_t issued = 0, retired = 0;
-    bool more = true;
-    auto issue = [&]() {
-        BulkJob j;
-        if (!bulk_next_chunk(p, i, x, xe, j)) {
-            more = false;
-            return;
-        }
-        const int s = int(issued % kStages);
-        jobs[s] = j;
-        const uint32_t announced = j.bytes + (p.stall_first && issued == 0 ? 16u : 0u);
-        bulk_load(ring_s + uint32_t(s) * kChunk, j.src, j.bytes, bar_s + 8 * s, announced, pol);
-        ++issued;
-    };
-    while (more && issued < kStages - 1) issue();
+    uint64_t k = 0;
     bool ok = true;
-    while (retired < issued) {
-        const int s = int(retired % kStages);
-        if (!mbar_wait_bounded(bar_s + 8 * s, (parity >> s) & 1u, kWaitNs)) {
+    for (;; ++k) {
+        const int s = int(k % kStages);
+        if (k >= uint64_t(kStages) &&
+            !mbar_wait_bounded(empty_s + 8 * s, uint32_t((k / kStages - 1) & 1), kWaitNs)) {
             ok = false;
             break;
         }
-        parity ^= 1u << s;
+        BulkJob j;
+        if (!bulk_next_chunk(p, i, x, xe, j)) {
+            r.jobs[s].bytes = 0;            // end of the range
+            mbar_arrive(full_s + 8 * s);
+            break;
+        }
+        r.jobs[s] = j;
+        const uint32_t announced = j.bytes + (p.stall_first && k == 0 ? 16u : 0u);
+        bulk_load(ring_s + uint32_t(s) * kChunk, j.src, j.bytes, full_s + 8 * s, announced, pol);
+    }
+    if (!ok) {
+        bulk_fault(p);
+        // the loads of the last kStages chunks may still be landing in shared memory
+        const uint64_t first = k > uint64_t(kStages) ? k - kStages : 0;
+        for (uint64_t c = first; c < k; ++c)
+            mbar_wait_bounded(full_s + 8 * int(c % kStages), uint32_t((c / kStages) & 1), kDrainNs);
+    }
+}
+
+__device__ void bulk_consume(const CopyParams& p, uint32_t ring_s, BulkRing& r) {
+    const uint32_t full_s = smem_addr(r.full), empty_s = smem_addr(r.empty);
+    const uint64_t pol = evict_first_policy();
+    for (uint64_t k = 0;; ++k) {
+        const int s = int(k % kStages);
+        if (!mbar_wait_bounded(full_s + 8 * s, uint32_t((k / kStages) & 1), kWaitNs)) {
+            bulk_fault(p);
+            break;
+        }
+        const BulkJob j = r.jobs[s];
+        if (j.bytes == 0) break;
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        const BulkJob j = jobs[s];
         bulk_store(j.dst, ring_s + uint32_t(s) * kChunk, j.bytes, pol);
         if (j.dst2) bulk_store(j.dst2, ring_s + uint32_t(s) * kChunk, j.bytes, pol);
         asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-        ++retired;
-        if (more) {
-            // the buffer of chunk retired-2 is refilled: its store group,
-            // all but the newest, must have finished reading it
-            asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
-            issue();
-        }
-    }
-    if (!ok) {
-        if (p.fault) {
-            *reinterpret_cast<volatile uint32_t*>(p.fault) = 1u;
-            __threadfence_system();
-        }
-        // let the loads still in flight land before the CTA's shared memory goes away
-        for (; retired < issued; ++retired) {
-            const int s = int(retired % kStages);
-            mbar_wait_bounded(bar_s + 8 * s, (parity >> s) & 1u, kDrainNs);
-            parity ^= 1u << s;
+        if (k >= uint64_t(kLag)) {
+            // groups up to k - kLag have read their buffers: hand that one back
+            asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(kLag) : "memory");
+            mbar_arrive(empty_s + 8 * int((k - kLag) % kStages));
         }
     }
     asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
@@ -416,16 +439,24 @@ __device__ void bulk_drive(const CopyParams& p, int i, uint64_t x, uint64_t xe, 
 
 __global__ void __launch_bounds__(kCopyThreads, 1) copy_bulk_kernel(CopyParams p) {
     extern __shared__ __align__(128) uint8_t ring[];
-    __shared__ __align__(8) uint64_t bars[kStages];
-    __shared__ BulkJob jobs[kStages];
+    __shared__ __align__(8) BulkRing r;
     uint64_t x, xe;
     int first;
     if (!cta_range(p, x, xe, first)) return;
-    if (threadIdx.x < 32) {
-        if (threadIdx.x == 0) bulk_drive(p, first, x, xe, ring, bars, jobs);
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(smem_addr(&r.full[s]));
+            mbar_init(smem_addr(&r.empty[s]));
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+    if (threadIdx.x < 64) {
+        if (threadIdx.x == 0) bulk_produce(p, first, x, xe, smem_addr(ring), r);
+        else if (threadIdx.x == 32) bulk_consume(p, smem_addr(ring), r);
         return;
     }
-    walk_entries<kWorkers, true>(p, first, x, xe, int(threadIdx.x) - 32);
+    walk_entries<kWorkers, true>(p, first, x, xe, int(threadIdx.x) - 64);
 }
 
 }  // namespace
