@@ -94,10 +94,11 @@ def kernel_source_sha(files):
     return h.hexdigest()[:16]
 
 
-KERNEL_FILES = {"measure": ["lc_measure.cu", "lc_reduce.cuh", "lc_internal.cuh"],
+KERNEL_FILES = {"measure": ["lc_measure.cu", "lc_bulk.cuh", "lc_reduce.cuh", "lc_internal.cuh"],
+                "measure_threads": ["lc_measure.cu", "lc_bulk.cuh", "lc_reduce.cuh", "lc_internal.cuh"],
                 "fused_adamw": ["lc_adamw.cu", "lc_reduce.cuh", "lc_internal.cuh"],
-                "pack": ["lc_copy.cu", "lc_internal.cuh"],
-                "pack_threads": ["lc_copy.cu", "lc_internal.cuh"]}
+                "pack": ["lc_copy.cu", "lc_bulk.cuh", "lc_internal.cuh"],
+                "pack_threads": ["lc_copy.cu", "lc_bulk.cuh", "lc_internal.cuh"]}
 
 
 def profiled_traffic(kernel, workload, persisted_bytes=None):
@@ -550,7 +551,9 @@ def run_ours(args):
     measure_name = "fused_adamw" if fused else "measure"
     mean_persisted = statistics.mean(r["nbytes"] for r in recs)
     pack_name = "pack" if args.copy_engine == "bulk" else "pack_threads"
-    traffic, tsrc = profiled_traffic(measure_name if dominant == "measure" else pack_name,
+    measure_prof = ("measure_threads" if measure_name == "measure" and args.copy_engine != "bulk"
+                    else measure_name)
+    traffic, tsrc = profiled_traffic(measure_prof if dominant == "measure" else pack_name,
                                      args.workload, mean_persisted if dominant == "pack" else None)
     if fused and dominant == "pack":
         traffic, tsrc = None, None       # the pack profile is of bf16 weights
@@ -594,9 +597,6 @@ def run_ours(args):
         except OSError:
             pass
         cap = full if avail == 0 else min(full, int(avail * 0.6))
-        # the pinned destination holds one step (the log store is cleared
-        # after every step): room for twice the largest step of the device loop
-        cap = min(cap, int(max(r["nbytes"] for r in recs) * 2) + (64 << 20))
         if graph:
             # the replayed pack writes straight into pinned host memory
             store = None
@@ -621,6 +621,11 @@ def run_ours(args):
                "ms_per_step": 1e3 * e_s / len(e_recs),
                "d2h_GBps": d2h / (statistics.mean((r["host_s"] - r["decision_s"]) if not graph
                                                   else r["host_s"] for r in e_recs)) / 1e9,
+               # the host link and memory are shared with other jobs: single steps
+               # can stall for tens of ms, which the mean above includes
+               "d2h_GBps_median_step": statistics.median(
+                   r["nbytes"] / max(1e-9, (r["host_s"] - r["decision_s"]) if not graph else r["host_s"])
+                   for r in e_recs) / 1e9,
                "d2h_link_GBps_measured": link,
                "note": "weights, snapshot and moments are device-resident training state; the "
                        "step's only host traffic is the decision block and the persisted "

@@ -71,23 +71,26 @@ typedef enum { LC_BF16 = 0, LC_F32 = 1 } lc_dtype;
  *                      R <- W for every layer and Eq. 2 sums u_l over steps. */
 typedef enum { LC_DRIFT_SNAPSHOT = 0, LC_DRIFT_ACCUMULATE = 1 } lc_drift_mode;
 
-/* Kernel that moves packed, committed and restored bytes (the bytes are the
- * same either way).
- * LC_COPY_BULK   : the bulk-copy engine (cp.async.bulk through shared
- *                  memory, one load-issuing and one store-issuing thread per
- *                  SM) whenever every address of the copy is device memory
- *                  -- segments, staging ring and destination -- else as
- *                  LC_COPY_THREADS (default).
- * LC_COPY_THREADS: every thread loads and stores 16-byte vectors. */
+/* How the kernels move bytes (the results are the same either way).
+ * LC_COPY_BULK   : the bulk-copy engine (cp.async.bulk through shared-memory
+ *                  rings, one load-issuing thread per SM) whenever every
+ *                  address involved is device memory: the pack, commit and
+ *                  restore copies (segments, staging ring and destination),
+ *                  and in LC_DRIFT_SNAPSHOT mode the measure's reads of W and
+ *                  R.  Otherwise as LC_COPY_THREADS (default).
+ * LC_COPY_THREADS: every thread loads (and stores) 16-byte vectors. */
 typedef enum { LC_COPY_BULK = 0, LC_COPY_THREADS = 1 } lc_copy_engine;
 
-/* LC_DEBUG_BULK_STALL: every bulk-engine copy launch waits for 16 bytes that
- * never arrive, once per CTA.  The engine's bounded wait (1 s) runs out, the
- * launch sets the context's copy-fault word and returns without finishing
- * its bytes, and the next call that checks the word (lc_select,
- * lc_wait_durable, lc_step_wait, lc_restore) fails with LC_ERR_TIMEOUT for
- * good.  It exists to test that path; it faults and hangs nothing. */
+/* Test switches of the bulk engine's bounded waits (they fault and hang
+ * nothing).  With one set, each CTA of the kernel named waits for 16 bytes
+ * that never arrive: the wait gives up after 1 s, the kernel sets the
+ * context's fault word and returns without finishing its work, and from
+ * then on lc_select, lc_wait_durable, lc_step_wait and lc_restore fail with
+ * LC_ERR_TIMEOUT.
+ * LC_DEBUG_BULK_STALL   : the pack / commit / restore copy kernel.
+ * LC_DEBUG_MEASURE_STALL: the bulk-load measure kernel. */
 #define LC_DEBUG_BULK_STALL 1
+#define LC_DEBUG_MEASURE_STALL 2
 
 /* One parameter tensor ("segment") of a layer (§2.2: embed_tokens, each
  * transformer block, the final norm and lm_head are the layers; a layer
@@ -126,7 +129,7 @@ typedef struct {
     uint64_t staging_bytes;  /* device staging ring used by lc_pack_async and
                                 lc_restore, split in two slots (default 512 MiB) */
     int32_t copy_engine;     /* lc_copy_engine (default LC_COPY_BULK)            */
-    int32_t debug_flags;     /* 0, or LC_DEBUG_BULK_STALL (tests only)           */
+    int32_t debug_flags;     /* 0, or LC_DEBUG_* switches (tests only)           */
 } lc_config;
 
 typedef struct lc_ctx lc_ctx;
@@ -162,6 +165,7 @@ typedef struct {
     uint64_t d2h_bytes;          /* bytes copied device -> host by the library  */
     uint64_t h2d_bytes;          /* bytes copied host -> device by the library  */
     int64_t bulk_copy_launches;  /* copy launches that ran on the bulk engine   */
+    int64_t bulk_measure_launches; /* measure launches on the bulk engine       */
 } lc_counters;
 
 /* Fills cfg with the defaults listed in lc_config. */

@@ -16,12 +16,13 @@ import os
 import numpy as np
 
 from . import _abi
-from ._abi import (LC_BF16, LC_COPY_BULK, LC_COPY_THREADS, LC_DEBUG_BULK_STALL,
+from ._abi import (LC_BF16, LC_COPY_BULK, LC_COPY_THREADS, LC_DEBUG_BULK_STALL, LC_DEBUG_MEASURE_STALL,
                    LC_DRIFT_ACCUMULATE, LC_DRIFT_SNAPSHOT, LC_F32, LCError, check, lc_config,
                    lc_counters, lc_segment, lc_select_info, lc_version)
 
 __all__ = ["LayerCheck", "Store", "LCError", "LC_BF16", "LC_F32", "LC_DRIFT_SNAPSHOT",
-           "LC_DRIFT_ACCUMULATE", "LC_DEBUG_BULK_STALL", "library", "segment", "crc32c",
+           "LC_DRIFT_ACCUMULATE", "LC_DEBUG_BULK_STALL", "LC_DEBUG_MEASURE_STALL", "library", "segment",
+           "crc32c",
            "manifest_read"]
 
 

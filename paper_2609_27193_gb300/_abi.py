@@ -24,6 +24,7 @@ LC_BF16, LC_F32 = 0, 1
 LC_DRIFT_SNAPSHOT, LC_DRIFT_ACCUMULATE = 0, 1
 LC_COPY_BULK, LC_COPY_THREADS = 0, 1
 LC_DEBUG_BULK_STALL = 1
+LC_DEBUG_MEASURE_STALL = 2
 
 
 class lc_segment(C.Structure):
@@ -64,7 +65,7 @@ class lc_counters(C.Structure):
     _fields_ = [("kernel_launches", C.c_int64), ("measure_launches", C.c_int64),
                 ("select_launches", C.c_int64), ("copy_launches", C.c_int64),
                 ("d2h_bytes", C.c_uint64), ("h2d_bytes", C.c_uint64),
-                ("bulk_copy_launches", C.c_int64)]
+                ("bulk_copy_launches", C.c_int64), ("bulk_measure_launches", C.c_int64)]
 
 
 class lc_manifest_record(C.Structure):

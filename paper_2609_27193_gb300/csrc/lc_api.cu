@@ -179,6 +179,9 @@ struct lc_ctx {
     // device memory
     void* d_tables = nullptr;
     MeasureParams mp{};
+    MeasureParams mpb{};                   // bulk-load measure: its own partition and partials
+    int measure_bulk_grid = 0;
+    bool bulk_measure = false;             // lc_measure takes the bulk-load kernel
     SelectParams sp{};
     CopyDesc* d_pack_desc = nullptr;
     CopyDesc* d_commit_desc = nullptr;
@@ -255,6 +258,19 @@ cudaError_t launch_copy_engine(lc_ctx* ctx, CopyParams p, bool bulk, uint64_t un
     return bulk ? launch_copy_bulk(p, grid, s) : launch_copy(p, grid, s);
 }
 
+// The Eq. 1 scan on the context's engine.
+lc_status launch_measure_engine(lc_ctx* ctx, cudaStream_t s) {
+    if (ctx->bulk_measure) {
+        LC_CUDA(launch_measure_bulk(ctx->mpb, ctx->measure_bulk_grid, s));
+        ctx->counters.bulk_measure_launches += 1;
+    } else {
+        LC_CUDA(launch_measure(ctx->mp, ctx->measure_grid, ctx->cfg.mode == LC_DRIFT_ACCUMULATE, s));
+    }
+    ctx->counters.kernel_launches += 1;
+    ctx->counters.measure_launches += 1;
+    return LC_OK;
+}
+
 }  // namespace
 
 // ---------------------------------------------------------------------------
@@ -294,7 +310,7 @@ extern "C" lc_status lc_create(lc_ctx** out, int device, void* cuda_stream, cons
         return fail(LC_ERR_INVALID_ARG, "lc_create: staging_bytes must be >= 2 MiB");
     if (c.copy_engine != LC_COPY_THREADS && c.copy_engine != LC_COPY_BULK)
         return fail(LC_ERR_INVALID_ARG, "lc_create: unknown copy engine %d", c.copy_engine);
-    if (c.debug_flags & ~LC_DEBUG_BULK_STALL)
+    if (c.debug_flags & ~(LC_DEBUG_BULK_STALL | LC_DEBUG_MEASURE_STALL))
         return fail(LC_ERR_INVALID_ARG, "lc_create: unknown debug flags 0x%x", unsigned(c.debug_flags));
     int ndev = 0;
     LC_CUDA(cudaGetDeviceCount(&ndev));
@@ -484,36 +500,53 @@ extern "C" lc_status lc_register_layout(lc_ctx* ctx, const lc_segment* segs, int
         d.vec_begin = V;
         V += d.nvec;
     }
-    int occ = 0;
-    LC_CUDA(measure_occupancy(&occ));
-    if (occ <= 0) occ = 1;
-    const int64_t ngran_all = (V + LC_MEASURE_ALIGN_VECS - 1) / LC_MEASURE_ALIGN_VECS;
-    const int64_t G = std::min<int64_t>(ngran_all, int64_t(ctx->sms) * occ);
-    ctx->measure_grid = int(G);
-    std::vector<int64_t> cta_vec(G + 1);
-    std::vector<int32_t> cta_seg0(G), cta_slot0(G);
-    std::vector<int32_t> seg_slot_begin(nseg + 1, -1);
-    int32_t slot = 0, s = 0;
-    {
-        // equal shares of the work space in granules of LC_MEASURE_ALIGN_VECS
+    // CTA work ranges of the measure work space: G equal shares in granules
+    // of LC_MEASURE_ALIGN_VECS, and `per_run` partial slots for every
+    // (CTA, segment) run
+    struct Partition {
+        int64_t G = 0;
+        std::vector<int64_t> cta_vec;
+        std::vector<int32_t> cta_seg0, cta_slot0, seg_slot_begin;
+        int32_t nslots = 0;
+    };
+    auto partition = [&](int64_t grid, int32_t per_run) {
+        Partition pt;
         const int64_t gran = LC_MEASURE_ALIGN_VECS;
         const int64_t ngran = (V + gran - 1) / gran;
-        for (int64_t b = 0; b <= G; ++b) cta_vec[b] = std::min(V, ngran * b / G * gran);
-    }
-    for (int64_t b = 0; b < G; ++b) {
-        const int64_t v0 = cta_vec[b], v1 = cta_vec[b + 1];
-        while (s < nseg && sd[s].vec_begin + sd[s].nvec <= v0) ++s;
-        cta_seg0[b] = s;
-        cta_slot0[b] = slot;
-        for (int32_t t = s; v0 < v1 && t < nseg && sd[t].vec_begin < v1; ++t) {
-            if (seg_slot_begin[t] < 0) seg_slot_begin[t] = slot;
-            ++slot;
+        pt.G = std::max<int64_t>(1, std::min<int64_t>(ngran, grid));
+        const int64_t G = pt.G;
+        pt.cta_vec.resize(G + 1);
+        pt.cta_seg0.resize(G);
+        pt.cta_slot0.resize(G);
+        pt.seg_slot_begin.assign(nseg + 1, -1);
+        for (int64_t b = 0; b <= G; ++b) pt.cta_vec[b] = std::min(V, ngran * b / G * gran);
+        int32_t slot = 0, s = 0;
+        for (int64_t b = 0; b < G; ++b) {
+            const int64_t v0 = pt.cta_vec[b], v1 = pt.cta_vec[b + 1];
+            while (s < nseg && sd[s].vec_begin + sd[s].nvec <= v0) ++s;
+            pt.cta_seg0[b] = s;
+            pt.cta_slot0[b] = slot;
+            for (int32_t t = s; v0 < v1 && t < nseg && sd[t].vec_begin < v1; ++t) {
+                if (pt.seg_slot_begin[t] < 0) pt.seg_slot_begin[t] = slot;
+                slot += per_run;
+            }
         }
-    }
-    seg_slot_begin[nseg] = slot;
-    for (int32_t t = nseg - 1; t >= 0; --t)
-        if (seg_slot_begin[t] < 0) seg_slot_begin[t] = seg_slot_begin[t + 1];
-    ctx->nslots = slot;
+        pt.seg_slot_begin[nseg] = slot;
+        for (int32_t t = nseg - 1; t >= 0; --t)
+            if (pt.seg_slot_begin[t] < 0) pt.seg_slot_begin[t] = pt.seg_slot_begin[t + 1];
+        pt.nslots = slot;
+        return pt;
+    };
+    int occ = 0;
+    LC_CUDA(measure_occupancy(&occ));
+    const Partition pa = partition(int64_t(ctx->sms) * std::max(1, occ), 1);
+    int bocc = 0;
+    LC_CUDA(measure_bulk_prepare(&bocc));
+    const Partition pb = partition(int64_t(ctx->sms) * std::max(1, bocc), kMeasureBulkSlotsPerRun);
+    const int64_t G = pa.G, Gb = pb.G;
+    ctx->measure_grid = int(G);
+    ctx->measure_bulk_grid = int(Gb);
+    ctx->nslots = pa.nslots;
 
     // packed layout: per layer all W sections, then exp_avg, then exp_avg_sq
     const uint64_t align = uint64_t(ctx->cfg.pack_align);
@@ -571,6 +604,12 @@ extern "C" lc_status lc_register_layout(lc_ctx* ctx, const lc_segment* segs, int
     const size_t o_segsum = tp.take(sizeof(double) * 2 * nseg);
     const size_t o_sums = tp.take(sizeof(double) * 3 * nlayers);
     const size_t o_ticket = tp.take(sizeof(unsigned int));
+    const size_t o_ctav_b = tp.take(sizeof(int64_t) * (Gb + 1));
+    const size_t o_ctas_b = tp.take(sizeof(int32_t) * Gb);
+    const size_t o_ctal_b = tp.take(sizeof(int32_t) * Gb);
+    const size_t o_segslot_b = tp.take(sizeof(int32_t) * (nseg + 1));
+    const size_t o_part_b = tp.take(sizeof(double2) * std::max(1, pb.nslots));
+    const size_t o_ticket_b = tp.take(sizeof(unsigned int));
     const size_t o_delta = tp.take(sizeof(double) * nlayers);
     const size_t o_tlast = tp.take(sizeof(int64_t) * nlayers);
     const size_t o_mult = tp.take(sizeof(double) * nlayers);
@@ -597,10 +636,14 @@ extern "C" lc_status lc_register_layout(lc_ctx* ctx, const lc_segment* segs, int
     }
     auto put = [&](size_t off, const void* src, size_t n) { if (n) std::memcpy(host.data() + off, src, n); };
     put(o_segs, sd.data(), sizeof(SegDev) * nseg);
-    put(o_ctav, cta_vec.data(), sizeof(int64_t) * (G + 1));
-    put(o_ctas, cta_seg0.data(), sizeof(int32_t) * G);
-    put(o_ctal, cta_slot0.data(), sizeof(int32_t) * G);
-    put(o_segslot, seg_slot_begin.data(), sizeof(int32_t) * (nseg + 1));
+    put(o_ctav, pa.cta_vec.data(), sizeof(int64_t) * (G + 1));
+    put(o_ctas, pa.cta_seg0.data(), sizeof(int32_t) * G);
+    put(o_ctal, pa.cta_slot0.data(), sizeof(int32_t) * G);
+    put(o_segslot, pa.seg_slot_begin.data(), sizeof(int32_t) * (nseg + 1));
+    put(o_ctav_b, pb.cta_vec.data(), sizeof(int64_t) * (Gb + 1));
+    put(o_ctas_b, pb.cta_seg0.data(), sizeof(int32_t) * Gb);
+    put(o_ctal_b, pb.cta_slot0.data(), sizeof(int32_t) * Gb);
+    put(o_segslot_b, pb.seg_slot_begin.data(), sizeof(int32_t) * (nseg + 1));
     put(o_lsb, ctx->layer_seg_begin.data(), sizeof(int32_t) * (nlayers + 1));
     put(o_mult, mult.data(), sizeof(double) * nlayers);
     put(o_lnumel, ctx->layer_numel.data(), sizeof(int64_t) * nlayers);
@@ -629,6 +672,19 @@ extern "C" lc_status lc_register_layout(lc_ctx* ctx, const lc_segment* segs, int
     mp.ticket = reinterpret_cast<unsigned int*>(base + o_ticket);
     mp.nseg = nseg;
     mp.nlayers = nlayers;
+    mp.fault = ctx->d_fault;
+    mp.stall_first = 0;
+    MeasureParams& mpb = ctx->mpb;
+    mpb = mp;
+    mpb.cta_vec_begin = reinterpret_cast<const int64_t*>(base + o_ctav_b);
+    mpb.cta_seg0 = reinterpret_cast<const int32_t*>(base + o_ctas_b);
+    mpb.cta_slot0 = reinterpret_cast<const int32_t*>(base + o_ctal_b);
+    mpb.seg_slot_begin = reinterpret_cast<const int32_t*>(base + o_segslot_b);
+    mpb.partials = reinterpret_cast<double2*>(base + o_part_b);
+    mpb.ticket = reinterpret_cast<unsigned int*>(base + o_ticket_b);
+    mpb.stall_first = (ctx->cfg.debug_flags & LC_DEBUG_MEASURE_STALL) ? 1 : 0;
+    ctx->bulk_measure = ctx->cfg.copy_engine == LC_COPY_BULK && ctx->cfg.mode == LC_DRIFT_SNAPSHOT &&
+                        all_device && !ctx->snap_missing;
 
     SelectParams& sp = ctx->sp;
     sp.sums = mp.sums;
@@ -690,9 +746,7 @@ extern "C" lc_status lc_measure(lc_ctx* ctx, int64_t step) {
     if (ctx->snap_missing)
         return fail(LC_ERR_STATE, "lc_measure: a segment has no snapshot (use lc_adamw_step_measure)");
     DeviceGuard g(ctx->device);
-    LC_CUDA(launch_measure(ctx->mp, ctx->measure_grid, ctx->cfg.mode == LC_DRIFT_ACCUMULATE, ctx->stream));
-    ctx->counters.kernel_launches += 1;
-    ctx->counters.measure_launches += 1;
+    LC_TRY(launch_measure_engine(ctx, ctx->stream));
     ctx->last_step = step;
     ctx->state = kMeasured;
     return LC_OK;
@@ -802,6 +856,7 @@ extern "C" lc_status lc_set_layer_sums_buffer(lc_ctx* ctx, double* sums_dev) {
     DeviceGuard g(ctx->device);
     LC_TRY(check_device_ptr(sums_dev, ctx->device, "lc_set_layer_sums_buffer", false));
     ctx->mp.sums = sums_dev;
+    ctx->mpb.sums = sums_dev;
     ctx->sp.sums = sums_dev;
     return LC_OK;
 }
@@ -1089,7 +1144,7 @@ lc_status check_step_dst(lc_ctx* ctx, void* dst, uint64_t capacity) {
 // Enqueues measure -> select -> pack -> commit -> decision readback on s.
 lc_status enqueue_step(lc_ctx* ctx, cudaStream_t s, int64_t step, bool step_from_counter, double tau,
                        int32_t max_staleness, uint8_t* dst, uint64_t capacity, uint8_t* host_block) {
-    LC_CUDA(launch_measure(ctx->mp, ctx->measure_grid, ctx->cfg.mode == LC_DRIFT_ACCUMULATE, s));
+    LC_TRY(launch_measure_engine(ctx, s));
     SelectParams p = ctx->sp;
     p.tau = tau;
     p.max_staleness = max_staleness;
@@ -1119,8 +1174,7 @@ lc_status enqueue_step(lc_ctx* ctx, cudaStream_t s, int64_t step, bool step_from
         LC_CUDA(launch_copy_engine(ctx, k, use_bulk(ctx, nullptr), UINT64_MAX, s));
     }
     LC_CUDA(cudaMemcpyAsync(host_block, ctx->d_result, ctx->rl.total, cudaMemcpyDeviceToHost, s));
-    ctx->counters.kernel_launches += 2;
-    ctx->counters.measure_launches += 1;
+    ctx->counters.kernel_launches += 1;
     ctx->counters.select_launches += 1;
     ctx->counters.d2h_bytes += ctx->rl.total;
     return LC_OK;

@@ -13,7 +13,7 @@
 // 16-byte aligned (the usual case: torch allocations, 256-byte packed
 // sections), else in the widest unit the three addresses share.  In GATHER
 // mode the padding of every section is written as zero.
-#include "lc_internal.cuh"
+#include "lc_bulk.cuh"
 
 namespace lc {
 namespace {
@@ -239,11 +239,6 @@ constexpr int kLag = LC_BULK_LAG;         // store groups still reading shared m
 constexpr int kWorkers = BS - 64;
 constexpr size_t kBulkSmem = size_t(kStages) * kChunk;
 static_assert(kChunk % 16 == 0 && kStages >= 2 && kLag >= 1 && kLag < kStages, "bulk ring shape");
-// A wait gives up after this long (a 32 KB load completes in microseconds);
-// the iteration cap bounds it even if the timer were not advancing.
-constexpr uint64_t kWaitNs = 1000000000ull;
-constexpr uint64_t kDrainNs = 100000000ull;
-constexpr uint32_t kWaitIters = 1u << 28;
 
 struct BulkJob {
     const uint8_t* src;
@@ -251,44 +246,6 @@ struct BulkJob {
     uint8_t* dst2;
     uint32_t bytes;
 };
-
-__device__ __forceinline__ uint32_t smem_addr(const void* p) {
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ uint64_t global_ns() {
-    uint64_t t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
-
-__device__ __forceinline__ void mbar_init(uint32_t bar) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar) : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-    uint32_t done;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(done)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    return done != 0;
-}
-
-// Waits for the phase with the given parity to complete, for at most
-// `limit_ns` (and kWaitIters polls).  Returns false if it gave up.
-__device__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
-    if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = global_ns();
-    for (uint32_t it = 0; it < kWaitIters; ++it) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if (global_ns() - t0 > limit_ns) return false;
-    }
-    return false;
-}
 
 // Every byte is read once and written once.  LC_BULK_L2_HINT asks L2 to
 // evict the copies' lines first: 0 never, 1 loads and stores, 2 loads only,
@@ -307,7 +264,7 @@ __device__ __forceinline__ uint64_t evict_first_policy() {
 
 __device__ __forceinline__ void bulk_load(uint32_t dst_smem, const void* src, uint32_t bytes, uint32_t bar,
                                           uint32_t announced, uint64_t pol) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(announced) : "memory");
+    mbar_expect_tx(bar, announced);
 #if LC_BULK_HINT_LOADS
     asm volatile(
         "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;"
@@ -315,10 +272,7 @@ __device__ __forceinline__ void bulk_load(uint32_t dst_smem, const void* src, ui
         : "memory");
 #else
     (void)pol;
-    asm volatile(
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst_smem),
-        "l"(src), "r"(bytes), "r"(bar)
-        : "memory");
+    bulk_g2s(dst_smem, src, bytes, bar);
 #endif
 }
 
@@ -365,17 +319,6 @@ __device__ bool bulk_next_chunk(const CopyParams& p, int& i, uint64_t& x, uint64
     return false;
 }
 
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-
-__device__ __forceinline__ void bulk_fault(const CopyParams& p) {
-    if (p.fault) {
-        *reinterpret_cast<volatile uint32_t*>(p.fault) = 1u;
-        __threadfence_system();
-    }
-}
-
 struct BulkRing {
     uint64_t full[kStages];
     uint64_t empty[kStages];
@@ -405,7 +348,7 @@ __device__ void bulk_produce(const CopyParams& p, int i, uint64_t x, uint64_t xe
         bulk_load(ring_s + uint32_t(s) * kChunk, j.src, j.bytes, full_s + 8 * s, announced, pol);
     }
     if (!ok) {
-        bulk_fault(p);
+        raise_fault(p.fault);
         // the loads of the last kStages chunks may still be landing in shared memory
         const uint64_t first = k > uint64_t(kStages) ? k - kStages : 0;
         for (uint64_t c = first; c < k; ++c)
@@ -419,7 +362,7 @@ __device__ void bulk_consume(const CopyParams& p, uint32_t ring_s, BulkRing& r) 
     for (uint64_t k = 0;; ++k) {
         const int s = int(k % kStages);
         if (!mbar_wait_bounded(full_s + 8 * s, uint32_t((k / kStages) & 1), kWaitNs)) {
-            bulk_fault(p);
+            raise_fault(p.fault);
             break;
         }
         const BulkJob j = r.jobs[s];
@@ -445,10 +388,10 @@ __global__ void __launch_bounds__(kCopyThreads, 1) copy_bulk_kernel(CopyParams p
     if (!cta_range(p, x, xe, first)) return;
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
-            mbar_init(smem_addr(&r.full[s]));
-            mbar_init(smem_addr(&r.empty[s]));
+            mbar_init(smem_addr(&r.full[s]), 1);
+            mbar_init(smem_addr(&r.empty[s]), 1);
         }
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        mbar_init_fence();
     }
     __syncthreads();
     if (threadIdx.x < 64) {

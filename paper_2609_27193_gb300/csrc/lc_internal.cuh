@@ -51,6 +51,11 @@ struct MeasureParams {
     unsigned int* ticket;            // CTA completion counter (reset by the last CTA)
     int32_t nseg;
     int32_t nlayers;
+    // bulk-load measure only: host-mapped fault word (a bounded wait ran
+    // out) and the test of that bound (each CTA's first load announces 16
+    // bytes more than it brings)
+    uint32_t* fault;
+    int32_t stall_first;
 };
 
 // One copy entry.  The entries of a launch tile a linear "work space"
@@ -184,6 +189,13 @@ struct AdamConsts {
 // Launchers (return the launch error, if any).
 cudaError_t launch_measure(const MeasureParams& p, int grid, bool write_ref, cudaStream_t s);
 cudaError_t measure_occupancy(int* blocks_per_sm);
+// Bulk-load measure: W and R stream through a shared-memory ring
+// (cp.async.bulk); its partition gives every (CTA, segment) run
+// kMeasureBulkSlotsPerRun consecutive partial slots.  W and R must be
+// device memory; snapshot mode only.
+constexpr int kMeasureBulkSlotsPerRun = kMeasureThreads / 32 - 1;
+cudaError_t launch_measure_bulk(const MeasureParams& p, int grid, cudaStream_t s);
+cudaError_t measure_bulk_prepare(int* blocks_per_sm);
 cudaError_t launch_adamw_measure(const MeasureParams& p, const OptSegDev* opt, const AdamConsts& c,
                                  int grid, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, cudaStream_t s);

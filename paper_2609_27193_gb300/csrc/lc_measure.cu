@@ -14,6 +14,7 @@
 // Precision: per-thread fp32 accumulators take at most kUnroll * kFlush
 // terms each before they are added (fixed tree) into per-thread fp64 sums;
 // the relative error of a layer sum is below about 2e-6 (all terms >= 0).
+#include "lc_bulk.cuh"
 #include "lc_reduce.cuh"
 
 namespace lc {
@@ -191,6 +192,200 @@ __global__ void __launch_bounds__(kMeasureThreads) measure_kernel(const MeasureP
     finalize(p);
 }
 
+// ---------------------------------------------------------------------------
+// Bulk-load measure.  The CTA's work range is the same walk over segment
+// runs as above, turned into a sequence of jobs by one producer thread
+// (warp 0): for the full co-aligned vectors of a run, chunks of up to
+// kMChunk bytes of W and the same bytes of R loaded by cp.async.bulk into a
+// ring of kMStages buffers (one "full" mbarrier per buffer, completed by the
+// loads' byte count); for partial edge vectors and runs whose W and R are
+// not co-aligned, a job the consumers read from global memory element by
+// element; after each run a flush.  Warps 1..7 consume every job in order:
+// each thread adds its 16-byte vectors of the chunk into fp32 lanes (at most
+// ceil(chunk vectors / 224) terms before they go to fp64), and at a flush
+// each warp reduces its threads' fp64 sums in a fixed order and writes them
+// to its own partial slot of the run, so no barrier spans warps.  Each warp
+// hands a buffer back on its "empty" mbarrier (7 arrivals).  Every wait is
+// bounded; a wait that runs out raises the fault word.  Warp-wide decisions
+// (the wait's outcome) are taken by lane 0 and broadcast, so the lanes of a
+// warp never part ways.
+// ---------------------------------------------------------------------------
+#ifndef LC_MEASURE_BULK_STAGES
+#define LC_MEASURE_BULK_STAGES 2
+#endif
+#ifndef LC_MEASURE_BULK_CHUNK
+#define LC_MEASURE_BULK_CHUNK 24576
+#endif
+constexpr int kMStages = LC_MEASURE_BULK_STAGES;
+constexpr uint32_t kMChunk = LC_MEASURE_BULK_CHUNK;      // bytes of W (and of R) per buffer
+constexpr int kMConsumerWarps = kMeasureBulkSlotsPerRun;
+constexpr int kMConsumers = 32 * kMConsumerWarps;
+constexpr size_t kMeasureBulkSmem = size_t(kMStages) * 2 * kMChunk;
+static_assert(kMChunk % 16 == 0 && kMStages >= 2, "measure ring shape");
+
+enum : int32_t { kJobChunk = 0, kJobScalar = 1, kJobFlush = 2, kJobEnd = 3 };
+
+struct MJob {
+    int64_t k0, k1;     // vectors [k0, k1) of the segment (chunk or scalar job)
+    int32_t kind;
+    int32_t seg;
+    int32_t slot;       // first partial slot of the run (flush)
+    int32_t esz_log2;   // element size of the segment (chunk)
+};
+
+struct MRing {
+    uint64_t full[kMStages];
+    uint64_t empty[kMStages];
+    MJob jobs[kMStages];
+};
+
+__device__ void measure_produce(const MeasureParams& p, uint8_t* ring, MRing& r) {
+    const uint32_t ring_s = smem_addr(ring);
+    const uint32_t full_s = smem_addr(r.full), empty_s = smem_addr(r.empty);
+    const int b = blockIdx.x;
+    int64_t v0 = p.cta_vec_begin[b];
+    const int64_t v1 = p.cta_vec_begin[b + 1];
+    int s = p.cta_seg0[b];
+    int slot = p.cta_slot0[b];
+    uint64_t k = 0;
+    bool stall = p.stall_first != 0;
+    auto post = [&](const MJob& j, const SegDev& sd) -> bool {
+        const int st = int(k % kMStages);
+        if (k >= uint64_t(kMStages) &&
+            !mbar_wait_bounded(empty_s + 8 * st, uint32_t((k / kMStages - 1) & 1), kWaitNs))
+            return false;
+        r.jobs[st] = j;
+        if (j.kind == kJobChunk) {
+            const uint32_t bytes = uint32_t(j.k1 - j.k0) * 16u;
+            const uint8_t* wb = sd.w - (int64_t(sd.lead) << sd.esz_log2) + 16 * j.k0;
+            const uint8_t* rb = sd.r - (int64_t(sd.lead) << sd.esz_log2) + 16 * j.k0;
+            mbar_expect_tx(full_s + 8 * st, 2 * bytes + (stall ? 16u : 0u));
+            stall = false;
+            bulk_g2s(ring_s + uint32_t(st) * 2 * kMChunk, wb, bytes, full_s + 8 * st);
+            bulk_g2s(ring_s + uint32_t(st) * 2 * kMChunk + kMChunk, rb, bytes, full_s + 8 * st);
+        } else {
+            mbar_arrive(full_s + 8 * st);
+        }
+        ++k;
+        return true;
+    };
+    bool ok = true;
+    SegDev sd{};
+    while (ok && v0 < v1 && s < p.nseg) {
+        sd = p.segs[s];
+        const int64_t seg_end = sd.vec_begin + sd.nvec;
+        const int64_t lo = v0 - sd.vec_begin;
+        const int64_t hi = (v1 < seg_end ? v1 : seg_end) - sd.vec_begin;
+        const int ve = 16 >> sd.esz_log2;
+        const bool head_partial = sd.lead > 0;
+        const bool tail_partial = ((int64_t(sd.lead) + sd.numel) % ve) != 0;
+        if (sd.coaligned) {
+            if (head_partial && lo <= 0 && 0 < hi) ok = post({0, 1, kJobScalar, s, slot, 0}, sd);
+            const int64_t kf0 = head_partial ? 1 : 0;
+            const int64_t kf1 = tail_partial ? sd.nvec - 1 : sd.nvec;
+            const int64_t a = lo > kf0 ? lo : kf0;
+            const int64_t e = hi < kf1 ? hi : kf1;
+            constexpr int64_t kCV = kMChunk / 16;
+            for (int64_t x = a; ok && x < e; x += kCV)
+                ok = post({x, (x + kCV < e ? x + kCV : e), kJobChunk, s, slot, sd.esz_log2}, sd);
+            const int64_t last = sd.nvec - 1;
+            if (ok && tail_partial && last >= lo && last < hi && !(head_partial && last == 0))
+                ok = post({last, last + 1, kJobScalar, s, slot, 0}, sd);
+        } else {
+            ok = post({lo, hi, kJobScalar, s, slot, 0}, sd);
+        }
+        if (ok) ok = post({0, 0, kJobFlush, s, slot, 0}, sd);
+        slot += kMeasureBulkSlotsPerRun;
+        ++s;
+        v0 = sd.vec_begin + hi;
+    }
+    if (ok) ok = post({0, 0, kJobEnd, 0, 0, 0}, sd);
+    if (!ok) {
+        raise_fault(p.fault);
+        // the loads of the last kMStages jobs may still be landing in shared memory
+        const uint64_t first = k > uint64_t(kMStages) ? k - kMStages : 0;
+        for (uint64_t c = first; c < k; ++c)
+            mbar_wait_bounded(full_s + 8 * int(c % kMStages), uint32_t((c / kMStages) & 1), kDrainNs);
+    }
+}
+
+__device__ void measure_consume(const MeasureParams& p, const uint8_t* ring, MRing& r) {
+    const uint32_t full_s = smem_addr(r.full), empty_s = smem_addr(r.empty);
+    const int tid = int(threadIdx.x) - 32;
+    const int warp = tid >> 5, lane = tid & 31;
+    double dd = 0.0, da = 0.0;
+    for (uint64_t k = 0;; ++k) {
+        const int st = int(k % kMStages);
+        const uint32_t parity = uint32_t((k / kMStages) & 1);
+        int ok = 1;
+        if (lane == 0) ok = mbar_wait_bounded(full_s + 8 * st, parity, kWaitNs) ? 1 : 0;
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (!ok) {
+            if (lane == 0) raise_fault(p.fault);
+            break;
+        }
+        mbar_try_wait(full_s + 8 * st, parity);   // completed: orders this lane's reads after the loads
+        const MJob j = r.jobs[st];
+        if (j.kind == kJobEnd) break;
+        if (j.kind == kJobChunk) {
+            const uint4* W = reinterpret_cast<const uint4*>(ring + size_t(st) * 2 * kMChunk);
+            const uint4* R = W + kMChunk / 16;
+            const int n = int(j.k1 - j.k0);
+            float ad[8], aa[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) { ad[q] = 0.f; aa[q] = 0.f; }
+            if (j.esz_log2 == 1) {
+#pragma unroll 4
+                for (int v = tid; v < n; v += kMConsumers) accumulate<1>(W[v], R[v], ad, aa);
+            } else {
+#pragma unroll 4
+                for (int v = tid; v < n; v += kMConsumers) accumulate<2>(W[v], R[v], ad, aa);
+            }
+            dd += double(tree8(ad));
+            da += double(tree8(aa));
+        } else if (j.kind == kJobScalar) {
+            const SegDev sd = p.segs[j.seg];
+            for (int64_t v = j.k0 + tid; v < j.k1; v += kMConsumers) scalar_vector<false>(sd, v, dd, da);
+        } else {   // flush: this warp's share of the run, in a fixed order
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) {
+                dd += __shfl_down_sync(0xffffffffu, dd, off);
+                da += __shfl_down_sync(0xffffffffu, da, off);
+            }
+            if (lane == 0) p.partials[j.slot + warp] = make_double2(dd, da);
+            dd = 0.0;
+            da = 0.0;
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(empty_s + 8 * st);
+    }
+}
+
+__global__ void __launch_bounds__(kMeasureThreads, 1) measure_bulk_kernel(const MeasureParams p) {
+    extern __shared__ __align__(128) uint8_t ring[];
+    __shared__ __align__(8) MRing r;
+    __shared__ unsigned int s_ticket;
+    if (threadIdx.x == 0) {
+        for (int st = 0; st < kMStages; ++st) {
+            mbar_init(smem_addr(&r.full[st]), 1);
+            mbar_init(smem_addr(&r.empty[st]), kMConsumerWarps);
+        }
+        mbar_init_fence();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) measure_produce(p, ring, r);
+    else if (threadIdx.x >= 32) measure_consume(p, ring, r);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        s_ticket = atomicAdd(p.ticket, 1u);
+    }
+    __syncthreads();
+    if (s_ticket != gridDim.x - 1) return;
+    __threadfence();
+    finalize(p);
+}
+
 }  // namespace
 
 cudaError_t launch_measure(const MeasureParams& p, int grid, bool write_ref, cudaStream_t s) {
@@ -198,6 +393,20 @@ cudaError_t launch_measure(const MeasureParams& p, int grid, bool write_ref, cud
     if (write_ref) measure_kernel<true><<<grid, kMeasureThreads, 0, s>>>(p);
     else measure_kernel<false><<<grid, kMeasureThreads, 0, s>>>(p);
     return cudaGetLastError();
+}
+
+cudaError_t launch_measure_bulk(const MeasureParams& p, int grid, cudaStream_t s) {
+    cudaGetLastError();
+    measure_bulk_kernel<<<grid, kMeasureThreads, kMeasureBulkSmem, s>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t measure_bulk_prepare(int* blocks_per_sm) {
+    cudaError_t e = cudaFuncSetAttribute(measure_bulk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         int(kMeasureBulkSmem));
+    if (e != cudaSuccess) return e;
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, measure_bulk_kernel, kMeasureThreads,
+                                                         kMeasureBulkSmem);
 }
 
 cudaError_t measure_occupancy(int* blocks_per_sm) {

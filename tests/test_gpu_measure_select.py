@@ -31,7 +31,8 @@ def _bf16_vals(vals):
 # hand cases: exact sums, so u is bit-exact
 # ----------------------------------------------------------------------------
 
-def test_hand_cases_exact():
+@pytest.mark.parametrize("engine", ["bulk", "threads"])
+def test_hand_cases_exact(engine):
     torch = require_gpu()
     eps = 1e-8
     # H1 layer A, H1 layer B, H3 (two tensors), H2
@@ -41,7 +42,7 @@ def test_hand_cases_exact():
             4: ([0, 2.0 ** -10], [0, 0])}
     for k, (w, r) in vals.items():
         st.set_values(k, w=_bf16_vals(w), r=_bf16_vals(r))
-    lc = make_lc(st, eps_w=eps)
+    lc = make_lc(st, eps_w=eps, copy_engine=engine)
     sums = torch.zeros(3 * spec.nlayers, dtype=torch.float64, device="cuda")
     lc.set_layer_sums_buffer(sums)
     lc.measure(1)
@@ -57,6 +58,7 @@ def test_hand_cases_exact():
     assert u[3] == 2.0 ** -11 / eps
     # tau = 0.25 sits just above 0.25/(1+eps): only H2 persists
     assert mask.tolist() == [0, 0, 0, 1]
+    assert lc.counters()["bulk_measure_launches"] == (1 if engine == "bulk" else 0)
     lc.close()
 
 
@@ -67,9 +69,10 @@ def test_hand_cases_exact():
 EDGE_SIZES = [1, 7, 8, 9, 4095, 4096, (1 << 20) + 3, 33, 2, 100003]
 
 
+@pytest.mark.parametrize("engine", ["bulk", "threads"])
 @pytest.mark.parametrize("alloc", ["separate", "flat", "skew"])
 @pytest.mark.parametrize("dtype", ["bf16", "f32", "mixed"])
-def test_measure_edge_shapes(alloc, dtype):
+def test_measure_edge_shapes(alloc, dtype, engine):
     require_gpu()
     sizes = [(n, i % 4) for i, n in enumerate(EDGE_SIZES)]
     spec = custom_shape(sizes)
@@ -80,7 +83,7 @@ def test_measure_edge_shapes(alloc, dtype):
     st = gen.SyntheticState(spec, device="cuda", seed=5, alloc=alloc, dtypes=dts)
     scales = np.array([3e-3, 1e-2, 1e-4, 5e-2])
     st.drift(1, scales)
-    lc = make_lc(st)
+    lc = make_lc(st, copy_engine=engine)
     run = make_oracle(st)
     lc.measure(1)
     mask, u, _ = lc.select(1e-3, 100)
@@ -90,7 +93,8 @@ def test_measure_edge_shapes(alloc, dtype):
     lc.close()
 
 
-def test_measure_interleaved_registration_and_many_segments():
+@pytest.mark.parametrize("engine", ["bulk", "threads"])
+def test_measure_interleaved_registration_and_many_segments(engine):
     """Layer ids in any registration order; hundreds of uneven segments."""
     require_gpu()
     rng = np.random.default_rng(3)
@@ -103,7 +107,7 @@ def test_measure_interleaved_registration_and_many_segments():
     spec = custom_shape(sizes)
     st = gen.SyntheticState(spec, device="cuda", seed=8, alloc="flat")
     st.drift(1, gen.loguniform(37, 1e-4, 3e-2, rng))
-    lc = make_lc(st)
+    lc = make_lc(st, copy_engine=engine)
     run = make_oracle(st)
     lc.measure(1)
     mask, u, _ = lc.select(2e-3, 100)
@@ -113,11 +117,12 @@ def test_measure_interleaved_registration_and_many_segments():
     lc.close()
 
 
-def test_measure_deterministic_and_zero_drift():
+@pytest.mark.parametrize("engine", ["bulk", "threads"])
+def test_measure_deterministic_and_zero_drift(engine):
     torch = require_gpu()
     spec = shapes.tiny()
     st = gen.SyntheticState(spec, device="cuda", seed=1)
-    lc = make_lc(st)
+    lc = make_lc(st, copy_engine=engine)
     # W == R: every layer measures exactly 0 (Eq. 1 numerator)
     lc.measure(1)
     mask, u, _ = lc.select(1e-3, 100)
@@ -301,3 +306,33 @@ def test_api_errors_and_state_machine():
     lc.measure(4)
     lc.select(1e-3, 100)
     lc.close()
+
+
+def test_bulk_measure_wait_bound_reports_timeout():
+    """LC_DEBUG_MEASURE_STALL: each CTA of the bulk-load measure waits for 16
+    bytes that never arrive; the waits give up after 1 s, the kernel returns,
+    and lc_select fails with LC_ERR_TIMEOUT instead of taking a decision
+    from incomplete sums.  A fresh context on the same device still works."""
+    import time
+    torch = require_gpu()
+    import paper_2609_27193_gb300 as P
+    spec = shapes.tiny()
+    st = gen.SyntheticState(spec, device="cuda", seed=2)
+    st.drift(1, np.full(spec.nlayers, 1e-2))
+    lc = make_lc(st, debug_flags=P.LC_DEBUG_MEASURE_STALL)
+    t0 = time.perf_counter()
+    lc.measure(1)
+    with pytest.raises(P.LCError) as e:
+        lc.select(1e-3, 100)
+    assert e.value.status == 6
+    assert time.perf_counter() - t0 < 30.0
+    assert lc.counters()["bulk_measure_launches"] == 1
+    lc.close()
+    lc2 = make_lc(st)
+    run = make_oracle(st)
+    lc2.measure(1)
+    mask, u, _ = lc2.select(1e-3, 100)
+    ou, _ = run.measure(st.host_all("W"))
+    run.select(ou, 1e-3, 100, 1)
+    compare_decision(mask, u, run, ou, 1e-3)
+    lc2.close()
