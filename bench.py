@@ -614,6 +614,7 @@ def run_ours(args):
             if i >= max(1, args.warmup):
                 e_recs.append(r)
                 e_bytes.append(mbytes + pack_bytes(r["mask"], payload, wbytes, fused_commit=not fused))
+        link_after = d2h_link_probe(torch, dev)
         e_s = sum(r["host_s"] for r in e_recs)
         d2h = statistics.mean(r["nbytes"] for r in e_recs)
         e2e = {"value": sum(e_bytes) / e_s / 1e9, "unit": "GB/s", "h2d_bytes_per_step": 0,
@@ -621,12 +622,14 @@ def run_ours(args):
                "ms_per_step": 1e3 * e_s / len(e_recs),
                "d2h_GBps": d2h / (statistics.mean((r["host_s"] - r["decision_s"]) if not graph
                                                   else r["host_s"] for r in e_recs)) / 1e9,
-               # the host link and memory are shared with other jobs: single steps
-               # can stall for tens of ms, which the mean above includes
-               "d2h_GBps_median_step": statistics.median(
-                   r["nbytes"] / max(1e-9, (r["host_s"] - r["decision_s"]) if not graph else r["host_s"])
-                   for r in e_recs) / 1e9,
+               # the host link and host memory are shared with other jobs on the
+               # machine: the same copy has measured 50-193 GB/s minutes apart, so
+               # the link is probed right before and right after the loop
                "d2h_link_GBps_measured": link,
+               "d2h_link_GBps_after": link_after,
+               "steps_d2h_ms": [round(1e3 * ((r["host_s"] - r["decision_s"]) if not graph else r["host_s"]), 3)
+                                for r in e_recs],
+               "steps_d2h_bytes": [int(r["nbytes"]) for r in e_recs],
                "note": "weights, snapshot and moments are device-resident training state; the "
                        "step's only host traffic is the decision block and the persisted "
                        "layers copied into %s" % ("pinned host memory by the replayed graph's pack"

@@ -68,16 +68,28 @@ __device__ __forceinline__ void block_sum(double& d, double& a, double* sd, doub
     __syncthreads();
 }
 
+// Run by the last CTA: one warp per segment adds the segment's partial
+// slots (lane l takes slots l, l+32, ... in order, then a fixed shuffle
+// tree), so a segment that spans many CTAs costs a few dependent loads per
+// lane instead of one per slot; then one thread per layer adds its segments.
 __device__ void finalize(const MeasureParams& p) {
-    for (int s = threadIdx.x; s < p.nseg; s += blockDim.x) {
+    const int lane = threadIdx.x & 31;
+    for (int s = threadIdx.x >> 5; s < p.nseg; s += blockDim.x >> 5) {
         double d = 0.0, a = 0.0;
-        for (int j = p.seg_slot_begin[s]; j < p.seg_slot_begin[s + 1]; ++j) {
+        for (int j = p.seg_slot_begin[s] + lane; j < p.seg_slot_begin[s + 1]; j += 32) {
             const double2 v = __ldcg(&p.partials[j]);
             d += v.x;
             a += v.y;
         }
-        p.seg_sums[2 * s] = d;
-        p.seg_sums[2 * s + 1] = a;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+            d += __shfl_down_sync(0xffffffffu, d, off);
+            a += __shfl_down_sync(0xffffffffu, a, off);
+        }
+        if (lane == 0) {
+            p.seg_sums[2 * s] = d;
+            p.seg_sums[2 * s + 1] = a;
+        }
     }
     __syncthreads();
     for (int l = threadIdx.x; l < p.nlayers; l += blockDim.x) {
