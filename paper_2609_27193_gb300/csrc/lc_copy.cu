@@ -225,7 +225,7 @@ __global__ void __launch_bounds__(kCopyThreads) copy_kernel(CopyParams p) {
 // two sides write disjoint bytes and never synchronise.
 // ---------------------------------------------------------------------------
 #ifndef LC_BULK_STAGES
-#define LC_BULK_STAGES 4
+#define LC_BULK_STAGES 3
 #endif
 #ifndef LC_BULK_CHUNK
 #define LC_BULK_CHUNK 32768
@@ -289,32 +289,46 @@ __device__ __forceinline__ void bulk_store(void* dst, uint32_t src_smem, uint32_
 #endif
 }
 
+// The producer's position: entry i, work position x, and entry i's
+// descriptor and addresses kept in registers (read once per entry, not once
+// per chunk).
+struct ChunkCursor {
+    int i;
+    uint64_t x;
+    int cached;          // entry whose descriptor is in d and e, or -1
+    CopyDesc d;
+    EntryAddr e;
+};
+
 // Next chunk (at most kChunk bytes) of 16-byte-aligned payload at or after
-// work position x, advancing x (and the entry index i) past it.  Takes
-// exactly the bytes copy_entry<..., true> leaves out.
-__device__ bool bulk_next_chunk(const CopyParams& p, int& i, uint64_t& x, uint64_t xe, BulkJob& j) {
-    while (x < xe && i < p.ndesc) {
-        const CopyDesc d = p.desc[i];
-        const uint64_t ent_end = d.woff + d.span;
-        if (ent_end <= x) {
-            ++i;
+// the cursor, advancing the cursor past it.  Takes exactly the bytes
+// copy_entry<..., true> leaves out.
+__device__ bool bulk_next_chunk(const CopyParams& p, ChunkCursor& c, uint64_t xe, BulkJob& j) {
+    while (c.x < xe && c.i < p.ndesc) {
+        if (c.cached != c.i) {
+            c.d = p.desc[c.i];
+            c.e = entry_addr(p, c.d);
+            c.cached = c.i;
+        }
+        const uint64_t ent_end = c.d.woff + c.d.span;
+        if (ent_end <= c.x) {
+            ++c.i;
             continue;
         }
         const uint64_t end = xe < ent_end ? xe : ent_end;
-        const uint64_t a = x - d.woff, b = end - d.woff;
-        const EntryAddr e = entry_addr(p, d);
-        const uint64_t pv = (b < d.nbytes ? b : d.nbytes) & ~uint64_t(15);
-        if (e.vec && a < pv) {
+        const uint64_t a = c.x - c.d.woff, b = end - c.d.woff;
+        const uint64_t pv = (b < c.d.nbytes ? b : c.d.nbytes) & ~uint64_t(15);
+        if (c.e.vec && a < pv) {
             const uint64_t n = pv - a < kChunk ? pv - a : kChunk;
-            j.src = e.src + a;
-            j.dst = e.dst + a;
-            j.dst2 = e.dst2 ? e.dst2 + a : nullptr;
+            j.src = c.e.src + a;
+            j.dst = c.e.dst + a;
+            j.dst2 = c.e.dst2 ? c.e.dst2 + a : nullptr;
             j.bytes = uint32_t(n);
-            x += n;
+            c.x += n;
             return true;
         }
-        x = end;
-        ++i;
+        c.x = end;
+        ++c.i;
     }
     return false;
 }
@@ -328,6 +342,12 @@ struct BulkRing {
 __device__ void bulk_produce(const CopyParams& p, int i, uint64_t x, uint64_t xe, uint32_t ring_s, BulkRing& r) {
     const uint32_t full_s = smem_addr(r.full), empty_s = smem_addr(r.empty);
     const uint64_t pol = evict_first_policy();
+    ChunkCursor c;
+    c.i = i;
+    c.x = x;
+    c.cached = -1;
+    BulkJob j;
+    bool have = bulk_next_chunk(p, c, xe, j);   // the next job is found before its buffer is free
     uint64_t k = 0;
     bool ok = true;
     for (;; ++k) {
@@ -337,8 +357,7 @@ __device__ void bulk_produce(const CopyParams& p, int i, uint64_t x, uint64_t xe
             ok = false;
             break;
         }
-        BulkJob j;
-        if (!bulk_next_chunk(p, i, x, xe, j)) {
+        if (!have) {
             r.jobs[s].bytes = 0;            // end of the range
             mbar_arrive(full_s + 8 * s);
             break;
@@ -346,6 +365,7 @@ __device__ void bulk_produce(const CopyParams& p, int i, uint64_t x, uint64_t xe
         r.jobs[s] = j;
         const uint32_t announced = j.bytes + (p.stall_first && k == 0 ? 16u : 0u);
         bulk_load(ring_s + uint32_t(s) * kChunk, j.src, j.bytes, full_s + 8 * s, announced, pol);
+        have = bulk_next_chunk(p, c, xe, j);
     }
     if (!ok) {
         raise_fault(p.fault);

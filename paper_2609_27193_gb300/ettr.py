@@ -118,7 +118,9 @@ def policies_from_bench(line, t_iter, h2d_gbps=None, restart=0.0, d2h_overlaps=T
     time) over the same link.  Both restart by reading the full state."""
     persisted = line["persisted_bytes_per_step"]
     link = (line.get("e2e") or {}).get("d2h_link_GBps_measured") or 193.0
-    full_bytes = persisted / max(line["selected_fraction"], 1e-9)
+    # every layer's block (the bench reports it; older lines: estimated from
+    # the persisted share of the layers)
+    full_bytes = line.get("full_state_bytes") or persisted / max(line["selected_fraction"], 1e-9)
     step_s = line["ms_per_step"] / 1e3
     d2h_s = persisted / (link * 1e9)
     # the D2H hides behind the next iteration up to t_iter when it overlaps

@@ -65,3 +65,7 @@ def test_policies_from_a_bench_line():
     assert pol["layercheck"].t_ckpt_segment == pytest.approx(0.012)     # D2H (0.1 s) hidden
     slow = E.policies_from_bench(line, t_iter=0.05, h2d_gbps=200.0)
     assert slow["layercheck"].t_ckpt_segment == pytest.approx(0.012 + 0.1 - 0.05)
+    # a reported full-state size takes precedence over the layer-share estimate
+    sized = E.policies_from_bench(dict(line, full_state_bytes=60e9), t_iter=2.0, h2d_gbps=200.0)
+    assert sized["full_d2h"] == pytest.approx(60e9 / 200e9)
+    assert sized["load"] == pytest.approx(0.3)
