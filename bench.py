@@ -60,6 +60,10 @@ def parse_args():
     ap.add_argument("--copy-engine", choices=["bulk", "threads"], default="bulk",
                     help="bulk: the bulk-copy engine through shared memory when every buffer is "
                          "device memory (default); threads: per-thread 16-byte vector copies")
+    ap.add_argument("--files", default=None, metavar="DIR",
+                    help="also append every e2e step's persisted versions to the checkpoint "
+                         "directory DIR (fsync'd), then time the metadata-driven recovery from it "
+                         "(lc_store_load_dir + lc_restore); DIR is removed afterwards")
     ap.add_argument("--lean", action="store_true",
                     help="no fp32 master weights in the generator (small case for kernel captures)")
     return ap.parse_args()
@@ -328,6 +332,36 @@ def reference_arm(args):
 # our arm
 # ---------------------------------------------------------------------------
 
+def files_recovery(P, lc, path, t_fail, written, write_s):
+    """§3.5 recovery from the checkpoint directory the e2e loop appended to:
+    the manifest picks each layer's newest version at or before t_fail and
+    only those blocks are read (CRC-checked), then lc_restore scatters them.
+    The directory's pages are dropped from the page cache first (its own
+    files only), so the reads come from the disk."""
+    import shutil
+    for name in ("manifest.lcm", "blocks.lcb"):
+        fd = os.open(os.path.join(path, name), os.O_RDONLY)
+        try:
+            os.posix_fadvise(fd, 0, 0, os.POSIX_FADV_DONTNEED)
+        finally:
+            os.close(fd)
+    recs, _, _, _ = P.manifest_read(path, verify_blocks=False)
+    on_disk = os.path.getsize(os.path.join(path, "blocks.lcb"))
+    t0 = time.perf_counter()
+    store, steps = lc.load_dir(path, t_fail)
+    t1 = time.perf_counter()
+    lc.restore(store, t_fail)
+    t2 = time.perf_counter()
+    loaded = sum(lc.layer_block_bytes(l) for l in range(len(steps)))
+    store.close()
+    shutil.rmtree(path, ignore_errors=True)
+    return {"records": len(recs), "block_bytes_on_disk": on_disk, "persisted_bytes": int(written),
+            "persist_GBps_fsync": written / write_s / 1e9 if write_s > 0 else None,
+            "load_dir_s": t1 - t0, "load_dir_GBps": loaded / (t1 - t0) / 1e9,
+            "restore_s": t2 - t1, "recovery_s": t2 - t0, "recovered_bytes": int(loaded),
+            "oldest_version_step": int(min(steps)), "t_fail": int(t_fail)}
+
+
 def d2h_link_probe(torch, dev, nbytes=4 << 30):
     """Plain device->pinned-host copy bandwidth measured beside the e2e loop
     (the host link is shared with other jobs on the machine, so it varies)."""
@@ -519,6 +553,7 @@ def run_ours(args):
     for _ in range(args.steps):
         t += 1
         recs.append(step(t, "device"))
+        recs[-1]["t"] = t
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
@@ -542,6 +577,26 @@ def run_ours(args):
         dist.all_reduce(tt, op=dist.ReduceOp.MAX)
         tot_bytes, tot_s = tb.item(), tt.item()
     value = tot_bytes / tot_s / 1e9
+    regimes = None
+    if wl.regimes:
+        # the drift regimes of the cadence workload, each summarised on its own
+        # (the last one, "sparse", persists about a tenth of the layers)
+        regimes = {}
+        for i, r in enumerate(recs):
+            name = cadence_scales(wl, shape, r["t"])[1]
+            g = regimes.setdefault(name, {"steps": 0, "sel": [], "bytes": [], "step_ms": [], "pack_ms": [],
+                                          "decision_ms": []})
+            g["steps"] += 1
+            g["sel"].append(float(r["mask"].mean()))
+            g["bytes"].append(r["nbytes"])
+            g["step_ms"].append(step_ms[i])
+            g["pack_ms"].append(pack_ms[i])
+            g["decision_ms"].append(decision_ms[i])
+        regimes = {n: {"steps": g["steps"], "selected_fraction": statistics.mean(g["sel"]),
+                       "persisted_GB_per_step": statistics.mean(g["bytes"]) / 1e9,
+                       "step_ms": statistics.mean(g["step_ms"]), "pack_ms": statistics.mean(g["pack_ms"]),
+                       "decision_ms_p50": statistics.median(g["decision_ms"])}
+                   for n, g in regimes.items()}
 
     hbm, peak_src = peaks()
     meas_gbs = mbytes / (statistics.mean(measure_ms) / 1e3) / 1e9
@@ -606,9 +661,23 @@ def run_ours(args):
             store = P.Store(lc, capacity_bytes=cap)
         link = d2h_link_probe(torch, dev)
         e_recs, e_bytes = [], []
+        f_bytes, f_s = 0, 0.0
+        files_note = None
+        if args.files and not graph:
+            import shutil
+            need = 1.3 * statistics.mean(r["nbytes"] for r in recs) * (max(1, args.warmup) + args.steps)
+            os.makedirs(args.files, exist_ok=True)
+            free = shutil.disk_usage(args.files).free
+            if need + (8 << 30) > free:
+                files_note = ("skipped: about %.0f GB would be written, %.0f GB free on %s"
+                              % (need / 1e9, free / 1e9, args.files))
         for i in range(max(1, args.warmup) + args.steps):
             t += 1
             r = step(t, "store", store)
+            if store is not None and args.files and files_note is None:
+                f0 = time.perf_counter()
+                f_bytes += store.persist_dir(args.files, sync=True)
+                f_s += time.perf_counter() - f0
             if store is not None:
                 store.clear()
             if i >= max(1, args.warmup):
@@ -636,6 +705,9 @@ def run_ours(args):
                                                   if graph else "the pinned store")}
         if store is not None:
             store.close()
+        if args.files and not graph:
+            e2e["files"] = ({"skipped": files_note} if files_note
+                            else files_recovery(P, lc, args.files, t, f_bytes, f_s))
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -671,6 +743,7 @@ def run_ours(args):
         "gpu_launches": int(c1["kernel_launches"] - c0["kernel_launches"]),
         "bulk_copy_launches": int(c1["bulk_copy_launches"] - c0["bulk_copy_launches"]),
         "capacity_overflow_steps": overflow,
+        "regimes": regimes,
         "clocks": clk, "timed_wall_s_with_input_generation": wall, "setup_s": setup_s,
     }
     if rank == 0:
