@@ -362,6 +362,34 @@ def files_recovery(P, lc, path, t_fail, written, write_s):
             "oldest_version_step": int(min(steps)), "t_fail": int(t_fail)}
 
 
+def restore_leg(torch, dev, P, lc, store, t, tau, full):
+    """§3.5 restore timed on its own: one step that persists every layer
+    (S_max = 0) into the cleared store, then lc_restore of that composite
+    (host -> device copies through the staging ring, scatter into W, m, v
+    and R), against a plain pinned host -> device copy probe."""
+    store.clear()
+    lc.measure(t)
+    lc.select(tau, 0)
+    lc.pack_async(store)
+    lc.commit_snapshot()
+    lc.wait_durable(t)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    lc.restore(store, t)
+    t1 = time.perf_counter()
+    h = torch.empty(4 << 30, dtype=torch.uint8, pin_memory=True)
+    d = torch.empty(4 << 30, dtype=torch.uint8, device=dev)
+    best = 0.0
+    for _ in range(3):
+        torch.cuda.synchronize()
+        a = time.perf_counter()
+        d.copy_(h, non_blocking=True)
+        torch.cuda.synchronize()
+        best = max(best, h.numel() / (time.perf_counter() - a) / 1e9)
+    del h, d
+    return {"bytes": int(full), "s": t1 - t0, "GBps": full / (t1 - t0) / 1e9, "h2d_link_GBps_measured": best}
+
+
 def d2h_link_probe(torch, dev, nbytes=4 << 30):
     """Plain device->pinned-host copy bandwidth measured beside the e2e loop
     (the host link is shared with other jobs on the machine, so it varies)."""
@@ -703,6 +731,9 @@ def run_ours(args):
                        "step's only host traffic is the decision block and the persisted "
                        "layers copied into %s" % ("pinned host memory by the replayed graph's pack"
                                                   if graph else "the pinned store")}
+        if store is not None and cap >= full:
+            e2e["restore"] = restore_leg(torch, dev, P, lc, store, t + 1, tau, full)
+            t += 1
         if store is not None:
             store.close()
         if args.files and not graph:

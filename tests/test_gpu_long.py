@@ -145,3 +145,76 @@ def test_cadence_regimes_with_failovers():
     assert regimes == set(wl.regimes)
     store.close()
     lc.close()
+
+
+def test_llama8b_fused_adamw_sampled_parity():
+    """The fused AdamW + drift step (§3.4.2) on the full Llama-3-8B layout in
+    the launch configuration `bench.py --path fused` times: fp32 master
+    weights as the optimizer's parameters, bf16 gradients and bf16 model
+    copies, accumulate mode.  For sampled transformer blocks the updated
+    weights, moments and model copies are bit-exact against the oracle's
+    AdamW, and u within 1e-5; the selection rule is re-checked on every
+    layer from the device's u, and sampled persisted blocks (fp32 weights
+    and moments) are compared byte for byte."""
+    torch = require_gpu()
+    import paper_2609_27193_gb300 as P
+    from lc_workloads.gen import mix_seed
+    hp = (1e-5, 0.9, 0.999, 1e-8, 0.01)
+    wl = WORKLOADS["8b"]
+    spec = wl.shape()
+    st = gen.SyntheticState(spec, device="cuda", seed=wl.seed, master=True, snapshot=False)
+    lc = P.LayerCheck(mode=P.LC_DRIFT_ACCUMULATE)
+    lc.register_layout([P.segment(t.layer, st.M[k], None, st.m[k], st.v[k])
+                        for k, t in enumerate(spec.tensors)], spec.nlayers)
+    grads = [torch.empty(t.numel, dtype=torch.bfloat16, device="cuda") for t in spec.tensors]
+    lc.register_optimizer(grads, st.W)
+    layer_tensors = [[k for k, t in enumerate(spec.tensors) if t.layer == l] for l in range(spec.nlayers)]
+    sample = [1, 16, 33]
+    delta = np.zeros(spec.nlayers)
+    t_last = np.zeros(spec.nlayers, dtype=np.int64)
+    tau, K = wl.tau, wl.max_staleness
+    host = gen.SyntheticState.to_numpy
+    for t in (1, 2):
+        g = torch.Generator(device="cuda")
+        for k, tsp in enumerate(spec.tensors):
+            g.manual_seed(mix_seed(wl.seed, t, k, 5))
+            grads[k].copy_(torch.randn(tsp.numel, generator=g, device="cuda").mul_(1e-3))
+        torch.cuda.synchronize()
+        ks = [k for l in sample for k in layer_tensors[l]]
+        P0 = {k: host(st.M[k]) for k in ks}
+        M0 = {k: host(st.m[k]) for k in ks}
+        V0 = {k: host(st.v[k]) for k in ks}
+        G = {k: host(grads[k]) for k in ks}
+        lc.adamw_step_measure(t, hp[0], beta1=hp[1], beta2=hp[2], eps=hp[3], weight_decay=hp[4])
+        mask, u, nbytes = lc.select(tau, K)
+        torch.cuda.synchronize()
+        for l in sample:
+            d_l = a_l = n_l = 0.0
+            for k in layer_tensors[l]:
+                model = np.zeros(spec.tensors[k].numel, np.uint16)
+                d, a = O.adamw_step(hp, t, P0[k], M0[k], V0[k], G[k], model)
+                d_l, a_l, n_l = d_l + d, a_l + a, n_l + spec.tensors[k].numel
+                assert np.array_equal(host(st.M[k]), P0[k]), "weights of tensor %d, step %d" % (k, t)
+                assert np.array_equal(host(st.m[k]), M0[k]), "exp_avg of tensor %d" % k
+                assert np.array_equal(host(st.v[k]), V0[k]), "exp_avg_sq of tensor %d" % k
+                assert np.array_equal(host(st.W[k]), model), "model copy of tensor %d" % k
+            ou = O.update_measure(d_l, a_l, n_l, 1e-8)
+            assert rel_err(u[l:l + 1], np.array([ou]))[0] <= U_RTOL, (l, t, u[l], ou)
+        omask, _, _ = O.select_step(u, delta, t_last, tau, K, t, O.ACCUMULATE)
+        assert np.array_equal(mask, omask), "select-only check at step %d" % t
+        dst = torch.empty(max(16, nbytes), dtype=torch.uint8, device="cuda")
+        lc.pack_device(dst)
+        lc.commit_snapshot()
+        torch.cuda.synchronize()
+        off = lc.offsets()
+        for l in sample:
+            if not mask[l]:
+                continue
+            ts = [O.Tensor(P0[k], None, M0[k], V0[k]) for k in layer_tensors[l]]
+            block = O.pack_layer(ts)
+            got = dst[int(off[l]):int(off[l]) + block.size].cpu().numpy()
+            assert np.array_equal(got, block), "block of layer %d at step %d" % (l, t)
+        del dst, P0, M0, V0, G
+    lc.close()
+    del st, grads
+    torch.cuda.empty_cache()
