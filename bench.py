@@ -57,6 +57,10 @@ def parse_args():
                     help="scan: measure against the snapshot (default); fused: AdamW step with "
                          "the drift read off the update, fp32 master weights; graph: the scan "
                          "step replayed as one captured CUDA graph with no host round trip")
+    ap.add_argument("--drift", choices=["snapshot", "accumulate"], default="snapshot",
+                    help="scan path: measure against the snapshot of each layer's last persistence "
+                         "(default), or against the previous step's weights with R <- W written "
+                         "every step (Eq. 1 literally; 6 B/param bf16)")
     ap.add_argument("--copy-engine", choices=["bulk", "threads"], default="bulk",
                     help="bulk: the bulk-copy engine through shared memory when every buffer is "
                          "device memory (default); threads: per-thread 16-byte vector copies")
@@ -458,7 +462,9 @@ def run_ours(args):
         # per-layer gradient bias: layers with consistent gradients move faster
         grad_bias = gen.u_shape(shape.nlayers, 2.0, 0.05, 0.3, np.random.default_rng(wl.seed + 7))
     else:
-        lc = P.LayerCheck(device=local, stream=side, copy_engine=args.copy_engine)
+        accumulate = args.drift == "accumulate"
+        lc = P.LayerCheck(device=local, stream=side, copy_engine=args.copy_engine,
+                          mode=P.LC_DRIFT_ACCUMULATE if accumulate else P.LC_DRIFT_SNAPSHOT)
         lc.register_layout([P.segment(t.layer, st.W[k], st.R[k], st.m[k], st.v[k])
                             for k, t in enumerate(shape.tensors)], shape.nlayers)
     sums = None
@@ -468,7 +474,9 @@ def run_ours(args):
     full = sum(lc.layer_block_bytes(l) for l in range(shape.nlayers))
     dst = torch.empty(full, dtype=torch.uint8, device=dev)
     payload, wbytes = layer_payload_bytes(st, fp32_weights=fused)
-    mbytes = fused_step_bytes(st) if fused else measure_bytes(st)
+    mbytes = fused_step_bytes(st) if fused else measure_bytes(st, accumulate=args.drift == "accumulate")
+    # the pack writes R <- W only in snapshot mode (accumulate mode's measure wrote it)
+    pack_commit = not fused and args.drift == "snapshot"
     gemm = None
     if args.workload == "8b-cadence":
         a = torch.randn(8192, 8192, device=dev, dtype=torch.bfloat16)
@@ -594,7 +602,7 @@ def run_ours(args):
     select_ms = [ms(r, 1, 2) for r in recs]
     pack_ms = [ms(r, 2, 3) for r in recs]
     decision_ms = [1e3 * r["decision_s"] for r in recs]
-    pbytes = [pack_bytes(r["mask"], payload, wbytes, fused_commit=not fused) for r in recs]
+    pbytes = [pack_bytes(r["mask"], payload, wbytes, fused_commit=pack_commit) for r in recs]
     tot_bytes = sum(mbytes + pb for pb in pbytes)
     tot_s = sum(step_ms) / 1e3
     frac_sel = float(np.mean([r["mask"].mean() for r in recs]))
@@ -710,7 +718,7 @@ def run_ours(args):
                 store.clear()
             if i >= max(1, args.warmup):
                 e_recs.append(r)
-                e_bytes.append(mbytes + pack_bytes(r["mask"], payload, wbytes, fused_commit=not fused))
+                e_bytes.append(mbytes + pack_bytes(r["mask"], payload, wbytes, fused_commit=pack_commit))
         link_after = d2h_link_probe(torch, dev)
         e_s = sum(r["host_s"] for r in e_recs)
         d2h = statistics.mean(r["nbytes"] for r in e_recs)
@@ -764,6 +772,7 @@ def run_ours(args):
                               if fused else "bf16 weights and snapshot, fp32 Adam moments; "
                               "arithmetic fp32 with fp64 combine"),
                    "copy_engine": args.copy_engine,
+                   "drift": "accumulate (fused AdamW)" if fused else args.drift,
                    "parallelism": "dp%d" % world},
         "decision_ms_p50": statistics.median(decision_ms),
         "decision_ms_p99": float(np.percentile(decision_ms, 99)),

@@ -261,7 +261,7 @@ cudaError_t launch_copy_engine(lc_ctx* ctx, CopyParams p, bool bulk, uint64_t un
 // The Eq. 1 scan on the context's engine.
 lc_status launch_measure_engine(lc_ctx* ctx, cudaStream_t s) {
     if (ctx->bulk_measure) {
-        LC_CUDA(launch_measure_bulk(ctx->mpb, ctx->measure_bulk_grid, s));
+        LC_CUDA(launch_measure_bulk(ctx->mpb, ctx->measure_bulk_grid, ctx->cfg.mode == LC_DRIFT_ACCUMULATE, s));
         ctx->counters.bulk_measure_launches += 1;
     } else {
         LC_CUDA(launch_measure(ctx->mp, ctx->measure_grid, ctx->cfg.mode == LC_DRIFT_ACCUMULATE, s));
@@ -683,8 +683,7 @@ extern "C" lc_status lc_register_layout(lc_ctx* ctx, const lc_segment* segs, int
     mpb.partials = reinterpret_cast<double2*>(base + o_part_b);
     mpb.ticket = reinterpret_cast<unsigned int*>(base + o_ticket_b);
     mpb.stall_first = (ctx->cfg.debug_flags & LC_DEBUG_MEASURE_STALL) ? 1 : 0;
-    ctx->bulk_measure = ctx->cfg.copy_engine == LC_COPY_BULK && ctx->cfg.mode == LC_DRIFT_SNAPSHOT &&
-                        all_device && !ctx->snap_missing;
+    ctx->bulk_measure = ctx->cfg.copy_engine == LC_COPY_BULK && all_device && !ctx->snap_missing;
 
     SelectParams& sp = ctx->sp;
     sp.sums = mp.sums;

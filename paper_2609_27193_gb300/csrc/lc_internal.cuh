@@ -192,9 +192,9 @@ cudaError_t measure_occupancy(int* blocks_per_sm);
 // Bulk-load measure: W and R stream through a shared-memory ring
 // (cp.async.bulk); its partition gives every (CTA, segment) run
 // kMeasureBulkSlotsPerRun consecutive partial slots.  W and R must be
-// device memory; snapshot mode only.
+// device memory.  write_ref: accumulate mode (R <- W as well).
 constexpr int kMeasureBulkSlotsPerRun = kMeasureThreads / 32 - 1;
-cudaError_t launch_measure_bulk(const MeasureParams& p, int grid, cudaStream_t s);
+cudaError_t launch_measure_bulk(const MeasureParams& p, int grid, bool write_ref, cudaStream_t s);
 cudaError_t measure_bulk_prepare(int* blocks_per_sm);
 cudaError_t launch_adamw_measure(const MeasureParams& p, const OptSegDev* opt, const AdamConsts& c,
                                  int grid, cudaStream_t s);

@@ -309,9 +309,13 @@ __device__ void measure_produce(const MeasureParams& p, uint8_t* ring, MRing& r)
     }
 }
 
+// Consumers: warps 1.. (warps 2.. in accumulate mode, where warp 1 writes R).
+template <bool WRITE_R>
 __device__ void measure_consume(const MeasureParams& p, const uint8_t* ring, MRing& r) {
+    constexpr int kFirstWarp = WRITE_R ? 2 : 1;
+    constexpr int kThreads = 32 * (kMeasureThreads / 32 - kFirstWarp);
     const uint32_t full_s = smem_addr(r.full), empty_s = smem_addr(r.empty);
-    const int tid = int(threadIdx.x) - 32;
+    const int tid = int(threadIdx.x) - 32 * kFirstWarp;
     const int warp = tid >> 5, lane = tid & 31;
     double dd = 0.0, da = 0.0;
     for (uint64_t k = 0;; ++k) {
@@ -336,16 +340,16 @@ __device__ void measure_consume(const MeasureParams& p, const uint8_t* ring, MRi
             for (int q = 0; q < 8; ++q) { ad[q] = 0.f; aa[q] = 0.f; }
             if (j.esz_log2 == 1) {
 #pragma unroll 4
-                for (int v = tid; v < n; v += kMConsumers) accumulate<1>(W[v], R[v], ad, aa);
+                for (int v = tid; v < n; v += kThreads) accumulate<1>(W[v], R[v], ad, aa);
             } else {
 #pragma unroll 4
-                for (int v = tid; v < n; v += kMConsumers) accumulate<2>(W[v], R[v], ad, aa);
+                for (int v = tid; v < n; v += kThreads) accumulate<2>(W[v], R[v], ad, aa);
             }
             dd += double(tree8(ad));
             da += double(tree8(aa));
         } else if (j.kind == kJobScalar) {
             const SegDev sd = p.segs[j.seg];
-            for (int64_t v = j.k0 + tid; v < j.k1; v += kMConsumers) scalar_vector<false>(sd, v, dd, da);
+            for (int64_t v = j.k0 + tid; v < j.k1; v += kThreads) scalar_vector<WRITE_R>(sd, v, dd, da);
         } else {   // flush: this warp's share of the run, in a fixed order
 #pragma unroll
             for (int off = 16; off > 0; off >>= 1) {
@@ -361,6 +365,39 @@ __device__ void measure_consume(const MeasureParams& p, const uint8_t* ring, MRi
     }
 }
 
+// Accumulate mode (R <- W after the measure, Eq. 1 against W(t-1)): one
+// thread stores every staged W chunk to R with a bulk store once the chunk
+// (and with it the old R) has landed, and hands the buffer back when the
+// store has read it.  Its partial slot of each run is written as zero.
+__device__ void measure_store_r(const MeasureParams& p, const uint8_t* ring, MRing& r) {
+    const uint32_t full_s = smem_addr(r.full), empty_s = smem_addr(r.empty);
+    const uint32_t ring_s = smem_addr(ring);
+    for (uint64_t k = 0;; ++k) {
+        const int st = int(k % kMStages);
+        if (!mbar_wait_bounded(full_s + 8 * st, uint32_t((k / kMStages) & 1), kWaitNs)) {
+            raise_fault(p.fault);
+            break;
+        }
+        const MJob j = r.jobs[st];
+        if (j.kind == kJobEnd) break;
+        if (j.kind == kJobChunk) {
+            const SegDev sd = p.segs[j.seg];
+            uint8_t* rb = sd.r - (int64_t(sd.lead) << sd.esz_log2) + 16 * j.k0;
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(rb),
+                         "r"(ring_s + uint32_t(st) * 2 * kMChunk), "r"(uint32_t(j.k1 - j.k0) * 16u)
+                         : "memory");
+            asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+            asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+        } else if (j.kind == kJobFlush) {
+            p.partials[j.slot + kMConsumerWarps - 1] = make_double2(0.0, 0.0);
+        }
+        mbar_arrive(empty_s + 8 * st);
+    }
+    asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+
+template <bool WRITE_R>
 __global__ void __launch_bounds__(kMeasureThreads, 1) measure_bulk_kernel(const MeasureParams p) {
     extern __shared__ __align__(128) uint8_t ring[];
     __shared__ __align__(8) MRing r;
@@ -373,8 +410,13 @@ __global__ void __launch_bounds__(kMeasureThreads, 1) measure_bulk_kernel(const 
         mbar_init_fence();
     }
     __syncthreads();
-    if (threadIdx.x == 0) measure_produce(p, ring, r);
-    else if (threadIdx.x >= 32) measure_consume(p, ring, r);
+    if (threadIdx.x == 0) {
+        measure_produce(p, ring, r);
+    } else if (WRITE_R && threadIdx.x < 64) {
+        if (threadIdx.x == 32) measure_store_r(p, ring, r);
+    } else if (threadIdx.x >= 32) {
+        measure_consume<WRITE_R>(p, ring, r);
+    }
     __syncthreads();
     if (threadIdx.x == 0) {
         __threadfence();
@@ -395,18 +437,22 @@ cudaError_t launch_measure(const MeasureParams& p, int grid, bool write_ref, cud
     return cudaGetLastError();
 }
 
-cudaError_t launch_measure_bulk(const MeasureParams& p, int grid, cudaStream_t s) {
+cudaError_t launch_measure_bulk(const MeasureParams& p, int grid, bool write_ref, cudaStream_t s) {
     cudaGetLastError();
-    measure_bulk_kernel<<<grid, kMeasureThreads, kMeasureBulkSmem, s>>>(p);
+    if (write_ref) measure_bulk_kernel<true><<<grid, kMeasureThreads, kMeasureBulkSmem, s>>>(p);
+    else measure_bulk_kernel<false><<<grid, kMeasureThreads, kMeasureBulkSmem, s>>>(p);
     return cudaGetLastError();
 }
 
 cudaError_t measure_bulk_prepare(int* blocks_per_sm) {
-    cudaError_t e = cudaFuncSetAttribute(measure_bulk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(measure_bulk_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          int(kMeasureBulkSmem));
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(measure_bulk_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 int(kMeasureBulkSmem));
     if (e != cudaSuccess) return e;
-    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, measure_bulk_kernel, kMeasureThreads,
-                                                         kMeasureBulkSmem);
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, measure_bulk_kernel<false>,
+                                                         kMeasureThreads, kMeasureBulkSmem);
 }
 
 cudaError_t measure_occupancy(int* blocks_per_sm) {

@@ -241,7 +241,7 @@ extern "C" lc_status lc_measure_noalloc(int device, void* cuda_stream, const lc_
         cudaGetLastError();
         return err(LC_ERR_CUDA, "lc_measure_noalloc: table upload failed: %s", cudaGetErrorString(e));
     }
-    MeasureParams p;
+    MeasureParams p{};
     p.segs = reinterpret_cast<const SegDev*>(ds.addr + kOffSegs);
     p.cta_vec_begin = reinterpret_cast<const int64_t*>(ds.addr + kOffCtaVec);
     p.cta_seg0 = reinterpret_cast<const int32_t*>(ds.addr + kOffCtaSeg);

@@ -68,13 +68,19 @@ def test_pack_device_bytes_and_fused_commit(align, alloc, engine):
     lc.close()
 
 
-def test_commit_unfused_and_accumulate_mode():
+@pytest.mark.parametrize("alloc", ["flat", "separate"])
+@pytest.mark.parametrize("engine", ["bulk", "threads"])
+def test_commit_unfused_and_accumulate_mode(engine, alloc):
+    """The unfused commit, and accumulate mode (the measure also writes
+    R <- W, Eq. 1 against W(t-1)) on both engines: flat buffers put every
+    tensor on an odd 16-byte offset, so partial edge vectors are written
+    element by element next to the bulk-stored interior."""
     torch = require_gpu()
     import paper_2609_27193_gb300 as P
     spec = shapes.tiny()
     for mode, fuse in ((P.LC_DRIFT_SNAPSHOT, False), (P.LC_DRIFT_ACCUMULATE, True)):
-        st = gen.SyntheticState(spec, device="cuda", seed=6, alloc="flat")
-        lc = make_lc(st, fuse_commit=fuse, mode=mode)
+        st = gen.SyntheticState(spec, device="cuda", seed=6, alloc=alloc)
+        lc = make_lc(st, fuse_commit=fuse, mode=mode, copy_engine=engine)
         run = make_oracle(st, mode=mode)
         scales = gen.loguniform(spec.nlayers, 1e-4, 1e-2, np.random.default_rng(1))
         for t in range(1, 7):
@@ -91,6 +97,7 @@ def test_commit_unfused_and_accumulate_mode():
             run.commit(run.last_mask, W)
             for k in range(len(spec.tensors)):
                 assert np.array_equal(st.host("R", k), run.R[k]), (mode, t, k)
+        assert lc.counters()["bulk_measure_launches"] == (6 if engine == "bulk" else 0)
         lc.close()
 
 
