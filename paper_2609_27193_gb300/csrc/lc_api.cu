@@ -15,6 +15,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <exception>
 #include <mutex>
 #include <set>
 #include <string>
@@ -403,8 +404,22 @@ struct TablePlan {
 
 }  // namespace
 
+static lc_status register_layout_impl(lc_ctx* ctx, const lc_segment* segs, int32_t nseg, int32_t nlayers,
+                                      const double* tau_mult);
+
+// The tables are host vectors sized by the layout: an allocation failure
+// is reported as LC_ERR_OOM rather than thrown across the C ABI.
 extern "C" lc_status lc_register_layout(lc_ctx* ctx, const lc_segment* segs, int32_t nseg,
                                         int32_t nlayers, const double* tau_mult) {
+    try {
+        return register_layout_impl(ctx, segs, nseg, nlayers, tau_mult);
+    } catch (const std::exception& e) {
+        return fail(LC_ERR_OOM, "lc_register_layout: %s", e.what());
+    }
+}
+
+static lc_status register_layout_impl(lc_ctx* ctx, const lc_segment* segs, int32_t nseg, int32_t nlayers,
+                                      const double* tau_mult) {
     g_err.clear();
     if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_register_layout: ctx is NULL");
     if (ctx->state != kNew) return fail(LC_ERR_STATE, "lc_register_layout: layout already registered");

@@ -16,6 +16,7 @@
 #include <algorithm>
 #include <atomic>
 #include <cstring>
+#include <exception>
 #include <set>
 #include <string>
 #include <thread>
@@ -285,7 +286,7 @@ extern "C" uint32_t lc_crc32c(const void* data, uint64_t nbytes, uint32_t crc) {
     return crc_parallel(static_cast<const uint8_t*>(data), nbytes, crc);
 }
 
-extern "C" lc_status lc_store_persist_dir(lc_store* st, const char* dir, int32_t sync, uint64_t* bytes_written) {
+static lc_status lc_store_persist_dir_impl(lc_store* st, const char* dir, int32_t sync, uint64_t* bytes_written) {
     const char* what = "lc_store_persist_dir";
     lc::set_last_error("");
     if (bytes_written) *bytes_written = 0;
@@ -357,9 +358,9 @@ extern "C" lc_status lc_store_persist_dir(lc_store* st, const char* dir, int32_t
     return LC_OK;
 }
 
-extern "C" lc_status lc_manifest_read(const char* dir, int32_t verify_blocks, lc_manifest_record* out, int64_t cap,
-                                      int64_t* n_out, int32_t* nlayers_out, uint32_t* layout_crc_out,
-                                      int32_t* torn_out) {
+static lc_status lc_manifest_read_impl(const char* dir, int32_t verify_blocks, lc_manifest_record* out,
+                                       int64_t cap, int64_t* n_out, int32_t* nlayers_out,
+                                       uint32_t* layout_crc_out, int32_t* torn_out) {
     const char* what = "lc_manifest_read";
     lc::set_last_error("");
     if (!dir) return fail_status(LC_ERR_INVALID_ARG, "%s: dir is NULL", what);
@@ -370,10 +371,17 @@ extern "C" lc_status lc_manifest_read(const char* dir, int32_t verify_blocks, lc
     if (rc != LC_OK) return rc;
     if (verify_blocks && !m.recs.empty()) {
         Fd blk(open(join(dir, "blocks.lcb").c_str(), O_RDONLY));
+        struct stat bs;
+        const uint64_t bsize = (blk.fd >= 0 && fstat(blk.fd, &bs) == 0) ? uint64_t(bs.st_size) : 0;
         std::vector<uint8_t> buf;
         for (auto& r : m.recs) {
+            // a record may name bytes the file does not have (a truncated file)
+            if (r.offset > bsize || r.bytes > bsize - r.offset) {
+                r.intact = 0;
+                continue;
+            }
             buf.resize(size_t(r.bytes));
-            r.intact = blk.fd >= 0 && read_all(blk.fd, buf.data(), r.bytes, r.offset) &&
+            r.intact = read_all(blk.fd, buf.data(), r.bytes, r.offset) &&
                        lc_crc32c(buf.data(), r.bytes, 0) == r.block_crc;
         }
     }
@@ -386,8 +394,8 @@ extern "C" lc_status lc_manifest_read(const char* dir, int32_t verify_blocks, lc
     return LC_OK;
 }
 
-extern "C" lc_status lc_store_load_dir(lc_ctx* ctx, const char* dir, int64_t t_fail, lc_store** out,
-                                       int64_t* layer_steps_out) {
+static lc_status lc_store_load_dir_impl(lc_ctx* ctx, const char* dir, int64_t t_fail, lc_store** out,
+                                        int64_t* layer_steps_out) {
     const char* what = "lc_store_load_dir";
     lc::set_last_error("");
     if (!ctx || !dir || !out) return fail_status(LC_ERR_INVALID_ARG, "%s: NULL argument", what);
@@ -466,4 +474,33 @@ extern "C" lc_status lc_store_load_dir(lc_ctx* ctx, const char* dir, int64_t t_f
     }
     *out = st;
     return LC_OK;
+}
+
+// The entry points: no C++ exception leaves the C ABI (a bad_alloc from a
+// vector sized by the layout or the manifest becomes LC_ERR_OOM).
+extern "C" lc_status lc_store_persist_dir(lc_store* st, const char* dir, int32_t sync, uint64_t* bytes_written) {
+    try {
+        return lc_store_persist_dir_impl(st, dir, sync, bytes_written);
+    } catch (const std::exception& e) {
+        return fail_status(LC_ERR_OOM, "lc_store_persist_dir: %s", e.what());
+    }
+}
+
+extern "C" lc_status lc_manifest_read(const char* dir, int32_t verify_blocks, lc_manifest_record* out, int64_t cap,
+                                      int64_t* n_out, int32_t* nlayers_out, uint32_t* layout_crc_out,
+                                      int32_t* torn_out) {
+    try {
+        return lc_manifest_read_impl(dir, verify_blocks, out, cap, n_out, nlayers_out, layout_crc_out, torn_out);
+    } catch (const std::exception& e) {
+        return fail_status(LC_ERR_OOM, "lc_manifest_read: %s", e.what());
+    }
+}
+
+extern "C" lc_status lc_store_load_dir(lc_ctx* ctx, const char* dir, int64_t t_fail, lc_store** out,
+                                       int64_t* layer_steps_out) {
+    try {
+        return lc_store_load_dir_impl(ctx, dir, t_fail, out, layer_steps_out);
+    } catch (const std::exception& e) {
+        return fail_status(LC_ERR_OOM, "lc_store_load_dir: %s", e.what());
+    }
 }

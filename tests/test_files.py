@@ -140,3 +140,19 @@ def test_manifest_errors(tmp_path, P):
     with pytest.raises(P.LCError) as e:
         P.manifest_read(str(d))
     assert e.value.status == 2
+
+
+def test_record_beyond_the_block_file_is_not_intact(tmp_path, P):
+    """A record whose CRC checks out but whose block lies past the end of a
+    truncated block file is reported not intact, without reading it."""
+    rng = np.random.default_rng(6)
+    layer_bytes = [4096, 8192]
+    vers = _versions(rng, layer_bytes, range(3))
+    d = str(tmp_path / "ckpt")
+    recs = F.write_dir(d, layer_bytes, vers)
+    blocks = os.path.join(d, "blocks.lcb")
+    with open(blocks, "r+b") as f:
+        f.truncate(recs[-1]["offset"] + 100)
+    got, _, _, torn = P.manifest_read(d, verify_blocks=True)
+    assert not torn and len(got) == len(recs)
+    assert [g["intact"] for g in got] == [1] * (len(recs) - 1) + [0]
