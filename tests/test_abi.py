@@ -107,6 +107,25 @@ def test_defaults_and_errors_without_gpu(lib):
     lib.lc_store_destroy(None)
 
 
+def test_config_validation_without_gpu(lib):
+    """lc_create checks its configuration before it touches a device."""
+    from paper_2609_27193_gb300 import _abi
+    cfg = _abi.lc_config()
+    lib.lc_config_default(C.byref(cfg))
+    assert cfg.copy_engine == _abi.LC_COPY_BULK and cfg.debug_flags == 0
+    ctx = C.c_void_p()
+    for field, value, word in (("copy_engine", 7, b"copy engine"), ("debug_flags", 8, b"debug flags"),
+                               ("timeout_ms", 0, b"timeout_ms"), ("staging_bytes", 1 << 20, b"staging_bytes")):
+        bad = _abi.lc_config()
+        lib.lc_config_default(C.byref(bad))
+        setattr(bad, field, value)
+        assert lib.lc_create(C.byref(ctx), 0, None, C.byref(bad)) == _abi.LC_ERR_INVALID_ARG, field
+        assert word in lib.lc_last_error(), (field, lib.lc_last_error())
+    import paper_2609_27193_gb300 as P
+    with pytest.raises(ValueError):
+        P.LayerCheck(copy_engine="tma")
+
+
 def test_product_path_has_no_fallback():
     """The package never imports the oracle, and fails loudly when the
     library is missing."""
