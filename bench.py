@@ -104,7 +104,8 @@ def kernel_source_sha(files):
 
 KERNEL_FILES = {"measure": ["lc_measure.cu", "lc_bulk.cuh", "lc_reduce.cuh", "lc_internal.cuh"],
                 "measure_threads": ["lc_measure.cu", "lc_bulk.cuh", "lc_reduce.cuh", "lc_internal.cuh"],
-                "fused_adamw": ["lc_adamw.cu", "lc_reduce.cuh", "lc_internal.cuh"],
+                "fused_adamw": ["lc_adamw.cu", "lc_bulk.cuh", "lc_reduce.cuh", "lc_internal.cuh"],
+                "fused_adamw_threads": ["lc_adamw.cu", "lc_bulk.cuh", "lc_reduce.cuh", "lc_internal.cuh"],
                 "pack": ["lc_copy.cu", "lc_bulk.cuh", "lc_internal.cuh"],
                 "pack_threads": ["lc_copy.cu", "lc_bulk.cuh", "lc_internal.cuh"]}
 
@@ -642,8 +643,7 @@ def run_ours(args):
     measure_name = "fused_adamw" if fused else "measure"
     mean_persisted = statistics.mean(r["nbytes"] for r in recs)
     pack_name = "pack" if args.copy_engine == "bulk" else "pack_threads"
-    measure_prof = ("measure_threads" if measure_name == "measure" and args.copy_engine != "bulk"
-                    else measure_name)
+    measure_prof = measure_name + ("_threads" if args.copy_engine != "bulk" else "")
     traffic, tsrc = profiled_traffic(measure_prof if dominant == "measure" else pack_name,
                                      args.workload, mean_persisted if dominant == "pack" else None)
     if fused and dominant == "pack":

@@ -183,6 +183,7 @@ struct lc_ctx {
     MeasureParams mpb{};                   // bulk-load measure: its own partition and partials
     int measure_bulk_grid = 0;
     bool bulk_measure = false;             // lc_measure takes the bulk-load kernel
+    bool bulk_adam = false;                // lc_adamw_step_measure takes the bulk-load kernel
     SelectParams sp{};
     CopyDesc* d_pack_desc = nullptr;
     CopyDesc* d_commit_desc = nullptr;
@@ -776,6 +777,7 @@ extern "C" lc_status lc_register_optimizer(lc_ctx* ctx, const lc_optim_segment* 
         return fail(LC_ERR_INVALID_ARG, "lc_register_optimizer: %d segments, the layout has %d", nseg, ctx->nseg);
     DeviceGuard g(ctx->device);
     std::vector<OptSegDev> od(ctx->nseg);
+    bool opt_device = true;
     for (int32_t pos = 0; pos < ctx->nseg; ++pos) {
         const int32_t i = ctx->order[pos];
         const lc_segment& s = ctx->segs[pos];
@@ -811,6 +813,13 @@ extern "C" lc_status lc_register_optimizer(lc_ctx* ctx, const lc_optim_segment* 
         if (o.model_copy) fast = fast && (uintptr_t(o.model_copy) - 2 * lead) % 8 == 0;
         (void)w0;
         d.fast = fast ? 1 : 0;
+        opt_device = opt_device && plain_device(o.grad) && (!o.model_copy || plain_device(o.model_copy));
+    }
+    // the bulk-load step: weights, moments, gradients and model copies all device memory
+    ctx->bulk_adam = ctx->cfg.copy_engine == LC_COPY_BULK && ctx->bulk_sources && opt_device;
+    if (ctx->bulk_adam) {
+        int occ = 0;
+        LC_CUDA(adamw_bulk_prepare(&occ));
     }
     if (!ctx->d_opt) {
         void* p = nullptr;
@@ -845,7 +854,12 @@ extern "C" lc_status lc_adamw_step_measure(lc_ctx* ctx, int64_t step, const lc_a
     c.rbc2 = float(1.0 / (1.0 - std::pow(hp->beta2, double(step))));
     c.eps = float(hp->eps);
     DeviceGuard g(ctx->device);
-    LC_CUDA(launch_adamw_measure(ctx->mp, ctx->d_opt, c, ctx->measure_grid, ctx->stream));
+    if (ctx->bulk_adam) {
+        LC_CUDA(launch_adamw_bulk(ctx->mpb, ctx->d_opt, c, ctx->measure_bulk_grid, ctx->stream));
+        ctx->counters.bulk_measure_launches += 1;
+    } else {
+        LC_CUDA(launch_adamw_measure(ctx->mp, ctx->d_opt, c, ctx->measure_grid, ctx->stream));
+    }
     ctx->counters.kernel_launches += 1;
     ctx->counters.measure_launches += 1;
     ctx->last_step = step;

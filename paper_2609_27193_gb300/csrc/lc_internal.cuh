@@ -198,6 +198,11 @@ cudaError_t launch_measure_bulk(const MeasureParams& p, int grid, bool write_ref
 cudaError_t measure_bulk_prepare(int* blocks_per_sm);
 cudaError_t launch_adamw_measure(const MeasureParams& p, const OptSegDev* opt, const AdamConsts& c,
                                  int grid, cudaStream_t s);
+// The fused step with its loads on the bulk engine: the bulk-load measure's
+// partition (kMeasureBulkSlotsPerRun slots per run); every array device memory.
+cudaError_t launch_adamw_bulk(const MeasureParams& p, const OptSegDev* opt, const AdamConsts& c, int grid,
+                              cudaStream_t s);
+cudaError_t adamw_bulk_prepare(int* blocks_per_sm);
 cudaError_t launch_select(const SelectParams& p, cudaStream_t s);
 cudaError_t launch_copy(const CopyParams& p, int grid, cudaStream_t s);
 cudaError_t copy_occupancy(int* blocks_per_sm);

@@ -70,11 +70,11 @@ class FusedState:
         return t.cpu().numpy().copy()
 
 
-def _run(sizes_layers, layout, grad_dtype, steps=4, tau=0.2, K=3):
+def _run(sizes_layers, layout, grad_dtype, steps=4, tau=0.2, K=3, engine="bulk"):
     torch = require_gpu()
     import paper_2609_27193_gb300 as P
     st = FusedState(sizes_layers, layout, grad_dtype)
-    lc = P.LayerCheck(mode=P.LC_DRIFT_ACCUMULATE)
+    lc = P.LayerCheck(mode=P.LC_DRIFT_ACCUMULATE, copy_engine=engine)
     lc.register_layout([P.segment(l, st.p[i], None, st.m[i], st.v[i])
                         for i, (_, l) in enumerate(st.specs)], st.nlayers)
     lc.register_optimizer(st.g, st.model)
@@ -125,6 +125,7 @@ def _run(sizes_layers, layout, grad_dtype, steps=4, tau=0.2, K=3):
             ts = [O.Tensor(P0[i], None, M0[i], V0[i]) for i, (_, ll) in enumerate(st.specs) if ll == l]
             block = O.pack_layer(ts)
             assert np.array_equal(got[int(off[l]):int(off[l]) + block.size], block), "block %d" % l
+    assert lc.counters()["bulk_measure_launches"] == (steps if engine == "bulk" else 0)
     lc.close()
     return mask
 
@@ -132,10 +133,16 @@ def _run(sizes_layers, layout, grad_dtype, steps=4, tau=0.2, K=3):
 SIZES = [(1, 0), (7, 0), (4095, 1), (4099, 1), (100003, 2), (65536, 3), (3, 3), (250001, 4)]
 
 
+@pytest.mark.parametrize("engine", ["bulk", "threads"])
 @pytest.mark.parametrize("layout", ["separate", "flat", "skew"])
 @pytest.mark.parametrize("grad_dtype", ["bf16", "f32"])
-def test_fused_adamw_bit_exact(layout, grad_dtype):
-    _run(SIZES, layout, grad_dtype)
+def test_fused_adamw_bit_exact(layout, grad_dtype, engine):
+    """Both engines: the bulk-load step takes chunks of 512 vectors of the
+    separate allocations (the 250,001- and 100,003-parameter segments span
+    several chunks and end in a partial vector); "flat" starts tensors on
+    odd offsets, so bf16 gradient vectors begin off 16 bytes and are peeled;
+    "skew" never lines up and goes element by element."""
+    _run(SIZES, layout, grad_dtype, engine=engine)
 
 
 def test_fused_step_requires_accumulate_mode_and_fp32_weights():
