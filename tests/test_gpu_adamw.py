@@ -172,3 +172,28 @@ def test_fused_step_requires_accumulate_mode_and_fp32_weights():
     lc.adamw_step_measure(1, 1e-3)
     lc.select(1e-3, 8)
     lc.close()
+
+
+def test_bulk_fused_step_wait_bound_reports_timeout():
+    """LC_DEBUG_MEASURE_STALL on the bulk-load fused step: each CTA's first
+    chunk announces 16 bytes that never arrive, the bounded waits run out,
+    and lc_select fails with LC_ERR_TIMEOUT; a fresh context still steps."""
+    import time
+    torch = require_gpu()
+    import paper_2609_27193_gb300 as P
+    st = FusedState([(250001, 0), (65536, 1)], "separate", "bf16")
+    lc = P.LayerCheck(mode=P.LC_DRIFT_ACCUMULATE, debug_flags=P.LC_DEBUG_MEASURE_STALL)
+    lc.register_layout([P.segment(l, st.p[i], None, st.m[i], st.v[i]) for i, (_, l) in enumerate(st.specs)],
+                       st.nlayers)
+    lc.register_optimizer(st.g, st.model)
+    st.new_grads(1)
+    t0 = time.perf_counter()
+    lc.adamw_step_measure(1, 1e-3)
+    with pytest.raises(P.LCError) as e:
+        lc.select(1e-3, 8)
+    assert e.value.status == 6
+    assert time.perf_counter() - t0 < 30.0
+    assert lc.counters()["bulk_measure_launches"] == 1
+    lc.close()
+    torch.cuda.synchronize()
+    _run([(4099, 0), (65536, 1)], "separate", "bf16", steps=2)
