@@ -58,33 +58,68 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectPara
     }
     __syncthreads();
 
-    if (threadIdx.x == 0) {
-        uint64_t run = 0, commit_work = 0;
-        int nsel = 0, nsec = 0, ncommit = 0;
-        int64_t mx = 0;
-        double num = 0.0, den = 0.0;
-        for (int l = 0; l < p.nlayers; ++l) {
-            const int64_t st = step - p.t_last[l];
-            mx = st > mx ? st : mx;
-            num = __dadd_rn(num, __dmul_rn(double(p.layer_numel[l]), double(st)));
-            den = __dadd_rn(den, double(p.layer_numel[l]));
-            if (mask[l]) {
-                off[l] = run;
-                run += p.layer_bytes[l];
-                scratch[3 * l] = nsec;
-                scratch[3 * l + 1] = ncommit;
-                scratch[3 * l + 2] = int64_t(commit_work);
+    // Stream layout and staleness statistics, layers ascending, in one
+    // thread so that the sums keep a fixed order; every per-layer input is
+    // first staged in shared memory by the whole CTA, a tile at a time, so
+    // the ordered loop reads no global memory.
+    __shared__ int64_t t_st[kSelectThreads];
+    __shared__ int64_t t_numel[kSelectThreads];
+    __shared__ uint64_t t_bytes[kSelectThreads];
+    __shared__ uint64_t t_cw[kSelectThreads];
+    __shared__ int32_t t_nsec[kSelectThreads];
+    __shared__ int32_t t_nwsec[kSelectThreads];
+    __shared__ uint8_t t_sel[kSelectThreads];
+    uint64_t run = 0, commit_work = 0;
+    int nsel = 0, nsec = 0, ncommit = 0;
+    int64_t mx = 0;
+    double num = 0.0, den = 0.0;
+    for (int base = 0; base < p.nlayers; base += kSelectThreads) {
+        const int l = base + int(threadIdx.x);
+        if (l < p.nlayers) {
+            const bool sel = mask[l] != 0;
+            t_st[threadIdx.x] = step - p.t_last[l];
+            t_numel[threadIdx.x] = p.layer_numel[l];
+            t_sel[threadIdx.x] = sel ? 1 : 0;
+            uint64_t cw = 0;
+            int ns = 0, nw = 0;
+            if (sel) {
                 const int s0 = p.layer_sec_begin[l];
-                nsec += p.layer_sec_begin[l + 1] - s0;
-                for (int j = s0; j < s0 + p.layer_wsec_count[l]; ++j) {
-                    commit_work += (p.secs[j].nbytes + 15) & ~uint64_t(15);
-                    ++ncommit;
+                ns = p.layer_sec_begin[l + 1] - s0;
+                nw = p.layer_wsec_count[l];
+                for (int j = s0; j < s0 + nw; ++j) cw += (p.secs[j].nbytes + 15) & ~uint64_t(15);
+            }
+            t_bytes[threadIdx.x] = sel ? p.layer_bytes[l] : 0;
+            t_cw[threadIdx.x] = cw;
+            t_nsec[threadIdx.x] = ns;
+            t_nwsec[threadIdx.x] = nw;
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            const int n = p.nlayers - base < kSelectThreads ? p.nlayers - base : kSelectThreads;
+            for (int i = 0; i < n; ++i) {
+                const int64_t st = t_st[i];
+                mx = st > mx ? st : mx;
+                num = __dadd_rn(num, __dmul_rn(double(t_numel[i]), double(st)));
+                den = __dadd_rn(den, double(t_numel[i]));
+                if (t_sel[i]) {
+                    off[base + i] = run;
+                    run += t_bytes[i];
+                    scratch[3 * (base + i)] = nsec;
+                    scratch[3 * (base + i) + 1] = ncommit;
+                    scratch[3 * (base + i) + 2] = int64_t(commit_work);
+                    nsec += t_nsec[i];
+                    ncommit += t_nwsec[i];
+                    commit_work += t_cw[i];
+                    ++nsel;
+                } else {
+                    off[base + i] = 0;
                 }
-                ++nsel;
-            } else {
-                off[l] = 0;
             }
         }
+        __syncthreads();
+    }
+
+    if (threadIdx.x == 0) {
         // a stream larger than the destination persists nothing this step
         const bool fits = run <= p.capacity;
         hdr->step = step;
