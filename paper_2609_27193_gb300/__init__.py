@@ -68,17 +68,29 @@ def _dtype_code(t):
 
 def segment(layer, w, snap, exp_avg=None, exp_avg_sq=None):
     """An lc_segment over torch CUDA tensors (contiguous, same numel); snap
-    may be None in accumulate mode (fused optimizer path only)."""
+    may be None in accumulate mode (fused optimizer path only).  The library
+    keeps raw pointers, so the segment holds references to the tensors and
+    the context that registers it keeps the segment."""
+    import torch
     for name, t in (("w", w), ("snap", snap), ("exp_avg", exp_avg), ("exp_avg_sq", exp_avg_sq)):
         if t is not None and not t.is_contiguous():
             raise ValueError("%s must be contiguous" % name)
+        if t is not None and t.device != w.device:
+            raise ValueError("%s must be on the device of w" % name)
     if snap is not None and (snap.dtype != w.dtype or snap.numel() != w.numel()):
         raise ValueError("snap must match w in dtype and size")
-    return lc_segment(int(layer), _dtype_code(w), w.data_ptr(),
-                      snap.data_ptr() if snap is not None else None,
-                      exp_avg.data_ptr() if exp_avg is not None else None,
-                      exp_avg_sq.data_ptr() if exp_avg_sq is not None else None,
-                      int(w.numel()))
+    if (exp_avg is None) != (exp_avg_sq is None):
+        raise ValueError("exp_avg and exp_avg_sq must both be given or both be None")
+    for name, t in (("exp_avg", exp_avg), ("exp_avg_sq", exp_avg_sq)):
+        if t is not None and (t.dtype != torch.float32 or t.numel() != w.numel()):
+            raise ValueError("%s must be float32 with the numel of w" % name)
+    s = lc_segment(int(layer), _dtype_code(w), w.data_ptr(),
+                   snap.data_ptr() if snap is not None else None,
+                   exp_avg.data_ptr() if exp_avg is not None else None,
+                   exp_avg_sq.data_ptr() if exp_avg_sq is not None else None,
+                   int(w.numel()))
+    s._refs = (w, snap, exp_avg, exp_avg_sq)
+    return s
 
 
 class LayerCheck:
@@ -142,6 +154,8 @@ class LayerCheck:
             self._keep.append(m)
         check(self._lib.lc_register_layout(self._ctx, arr, len(segments), int(nlayers), mult))
         self.nlayers = int(nlayers)
+        self._numels = [int(sg.numel) for sg in segments]
+        self._keep.append([getattr(sg, "_refs", None) for sg in segments])
 
     def measure(self, step):
         check(self._lib.lc_measure(self._ctx, int(step)))
@@ -149,11 +163,20 @@ class LayerCheck:
     def register_optimizer(self, grads, model_copies=None):
         """Gradients (and optional bf16 model copies) of every segment, in the
         order of register_layout, for the fused AdamW + drift step."""
+        import torch
         from ._abi import lc_optim_segment
         n = len(grads)
+        numels = getattr(self, "_numels", [])
+        if n != len(numels) or (model_copies is not None and len(model_copies) != n):
+            raise ValueError("need one gradient (and model copy) per registered segment")
         arr = (lc_optim_segment * n)()
         for i, g in enumerate(grads):
             mc = None if model_copies is None else model_copies[i]
+            if not g.is_contiguous() or g.numel() != numels[i]:
+                raise ValueError("gradient %d must be contiguous with the numel of its segment" % i)
+            if mc is not None and (mc.dtype != torch.bfloat16 or not mc.is_contiguous()
+                                   or mc.numel() != numels[i]):
+                raise ValueError("model copy %d must be contiguous bfloat16 with the numel of its segment" % i)
             arr[i] = lc_optim_segment(g.data_ptr(), _dtype_code(g), 0,
                                       mc.data_ptr() if mc is not None else None)
         self._keep.append((grads, model_copies))

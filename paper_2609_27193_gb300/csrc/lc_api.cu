@@ -24,6 +24,16 @@
 
 using namespace lc;
 
+// CTAs of a bulk-engine launch, in waves of one CTA per resident slot.  With
+// more than one wave each CTA takes a smaller share of the range, and SMs
+// that finish early start the next CTAs, which shortens the launch's tail.
+#ifndef LC_MEASURE_BULK_WAVES
+#define LC_MEASURE_BULK_WAVES 1
+#endif
+#ifndef LC_COPY_BULK_WAVES
+#define LC_COPY_BULK_WAVES 1
+#endif
+
 // ---------------------------------------------------------------------------
 // errors
 // ---------------------------------------------------------------------------
@@ -349,7 +359,7 @@ extern "C" lc_status lc_create(lc_ctx** out, int device, void* cuda_stream, cons
         lc_destroy(ctx);
         return fail(LC_ERR_CUDA, "lc_create: %s", cudaGetErrorString(e));
     }
-    ctx->bulk_grid = ctx->sms * std::max(1, bocc);
+    ctx->bulk_grid = ctx->sms * std::max(1, bocc) * LC_COPY_BULK_WAVES;
     *out = ctx;
     return LC_OK;
 }
@@ -558,7 +568,8 @@ static lc_status register_layout_impl(lc_ctx* ctx, const lc_segment* segs, int32
     const Partition pa = partition(int64_t(ctx->sms) * std::max(1, occ), 1);
     int bocc = 0;
     LC_CUDA(measure_bulk_prepare(&bocc));
-    const Partition pb = partition(int64_t(ctx->sms) * std::max(1, bocc), kMeasureBulkSlotsPerRun);
+    const Partition pb =
+        partition(int64_t(ctx->sms) * std::max(1, bocc) * LC_MEASURE_BULK_WAVES, kMeasureBulkSlotsPerRun);
     const int64_t G = pa.G, Gb = pb.G;
     ctx->measure_grid = int(G);
     ctx->measure_bulk_grid = int(Gb);
@@ -959,7 +970,7 @@ namespace {
 lc_status launch_copy_range(lc_ctx* ctx, const CopyDesc* desc, int ndesc, int mode, uint64_t lo,
                             uint64_t hi, uint8_t* base, cudaStream_t s) {
     if (hi <= lo || ndesc <= 0) return LC_OK;
-    CopyParams p;
+    CopyParams p{};
     p.desc = desc;
     p.ndesc = ndesc;
     p.mode = mode;
@@ -1022,6 +1033,8 @@ extern "C" lc_status lc_pack_async(lc_ctx* ctx, lc_store* st) {
         ctx->state = kPacked;
         return LC_OK;
     }
+    // the staging ring first: a failure leaves the store untouched
+    LC_TRY(ensure_staging(ctx));
     // reserve the destination of every selected layer block in the store
     struct Extent { uint64_t soff; uint8_t* host; uint64_t len; };
     std::vector<Extent> ext;
@@ -1057,7 +1070,6 @@ extern "C" lc_status lc_pack_async(lc_ctx* ctx, lc_store* st) {
             fresh.push_back({st->next_id++, l, 0, ctx->hdr.step, off, ctx->layer_bytes[l], slot});
         }
     }
-    LC_TRY(ensure_staging(ctx));
     // forget copies into this store that have completed
     st->inflight.erase(std::remove_if(st->inflight.begin(), st->inflight.end(),
                                       [](cudaEvent_t ev) {
@@ -1181,7 +1193,7 @@ lc_status enqueue_step(lc_ctx* ctx, cudaStream_t s, int64_t step, bool step_from
     p.capacity = capacity;
     LC_CUDA(launch_select(p, s));
     const ResultHeader* hdr_dev = reinterpret_cast<const ResultHeader*>(ctx->d_result);
-    CopyParams c;
+    CopyParams c{};
     c.desc = ctx->d_pack_desc;
     c.ndesc = 0;
     c.mode = kGather;

@@ -103,6 +103,22 @@ uint32_t crc_concat(uint32_t crc_a, uint32_t crc_b, uint64_t len_b) {
 
 uint32_t crc_serial(const uint8_t* p, uint64_t n, uint32_t crc) { return ~crc_feed(~crc, p, n); }
 
+// Runs `worker` on this thread and on up to n - 1 more.  The workers take
+// their items from one shared counter, so a thread that cannot be started
+// is simply left out (the others take its share) and no joinable thread is
+// abandoned while an exception unwinds.
+template <typename F>
+void run_on_threads(unsigned n, F&& worker) {
+    std::vector<std::thread> pool;
+    try {
+        pool.reserve(n);
+        for (unsigned t = 1; t < n; ++t) pool.emplace_back(worker);
+    } catch (const std::exception&) {
+    }
+    worker();
+    for (auto& t : pool) t.join();
+}
+
 // Pieces of kPiece bytes on up to hardware_concurrency threads, joined with
 // crc_concat.
 constexpr uint64_t kPiece = 64ull << 20;
@@ -119,11 +135,7 @@ uint32_t crc_parallel(const uint8_t* p, uint64_t n, uint32_t crc) {
             part[i] = crc_serial(p + a, b - a, 0);
         }
     };
-    const unsigned nthreads = unsigned(std::min<uint64_t>(hw, pieces));
-    std::vector<std::thread> pool;
-    for (unsigned t = 1; t < nthreads; ++t) pool.emplace_back(worker);
-    worker();
-    for (auto& t : pool) t.join();
+    run_on_threads(unsigned(std::min<uint64_t>(hw, pieces)), worker);
     for (uint64_t i = 0; i < pieces; ++i) {
         const uint64_t len = std::min(n, (i + 1) * kPiece) - i * kPiece;
         crc = crc_concat(crc, part[i], len);
@@ -331,7 +343,8 @@ static lc_status lc_store_persist_dir_impl(lc_store* st, const char* dir, int32_
     const int64_t nv = lc_store_num_versions(st);
     for (int64_t i = 0; i < nv; ++i) {
         lc_version v;
-        if (lc_store_get_version(st, i, &v) != LC_OK) return LC_ERR_STATE;
+        if (lc_store_get_version(st, i, &v) != LC_OK)
+            return fail_status(LC_ERR_STATE, "%s: version %lld of the store is unreadable", what, (long long)i);
         if (!v.durable || have.count({v.layer, v.step})) continue;
         lc_manifest_record r;
         r.layer = v.layer;
@@ -457,11 +470,7 @@ static lc_status lc_store_load_dir_impl(lc_ctx* ctx, const char* dir, int64_t t_
         }
     };
     const unsigned hw = std::max(1u, std::thread::hardware_concurrency());
-    const unsigned nthreads = unsigned(std::min<int64_t>(hw, nl));
-    std::vector<std::thread> pool;
-    for (unsigned t = 1; t < nthreads; ++t) pool.emplace_back(worker);
-    worker();
-    for (auto& t : pool) t.join();
+    run_on_threads(unsigned(std::min<int64_t>(hw, nl)), worker);
     for (int32_t l = 0; l < nl; ++l) {
         if (chosen[size_t(l)] < 0) {
             lc_store_destroy(st);

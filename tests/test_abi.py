@@ -137,3 +137,30 @@ def test_product_path_has_no_fallback():
                 assert "oracle" not in text.lower().replace("oracle-free", ""), f
     src = open(os.path.join(pkg, "_abi.py")).read()
     assert "raise ImportError" in src and "no CPU fallback" in src
+
+
+def test_segment_validation_without_gpu():
+    """The binding checks what a raw pointer cannot carry: moment dtypes and
+    sizes, contiguity, one device, and both moments or neither; a segment
+    keeps its tensors alive."""
+    torch = pytest.importorskip("torch")
+    import paper_2609_27193_gb300 as P
+    w = torch.zeros(8, dtype=torch.bfloat16)
+    r = torch.zeros(8, dtype=torch.bfloat16)
+    m = torch.zeros(8, dtype=torch.float32)
+    v = torch.zeros(8, dtype=torch.float32)
+    s = P.segment(0, w, r, m, v)
+    assert s.numel == 8 and s._refs[0] is w
+    bad = [
+        (w, r, m.to(torch.bfloat16), v),          # moments must be fp32
+        (w, r, m, v[:4]),                         # and as long as w
+        (w, r, m, None),                          # both or neither
+        (w, r[:4], m, v),                         # snapshot as long as w
+        (w, r.float(), m, v),                     # and of w's dtype
+        (w, torch.zeros(16, dtype=torch.bfloat16)[::2], m, v),   # contiguous
+    ]
+    for args in bad:
+        with pytest.raises(ValueError):
+            P.segment(0, *args)
+    with pytest.raises(TypeError):
+        P.segment(0, w.to(torch.float16), None, m, v)
