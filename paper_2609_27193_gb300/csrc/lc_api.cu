@@ -31,7 +31,7 @@ using namespace lc;
 #define LC_MEASURE_BULK_WAVES 1
 #endif
 #ifndef LC_COPY_BULK_WAVES
-#define LC_COPY_BULK_WAVES 1
+#define LC_COPY_BULK_WAVES 8
 #endif
 
 // ---------------------------------------------------------------------------
