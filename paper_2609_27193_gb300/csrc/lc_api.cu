@@ -9,6 +9,8 @@
 #include "lc_host.h"
 #include "lc_internal.cuh"
 
+#include <nvtx3/nvToolsExt.h>
+
 #include <algorithm>
 #include <chrono>
 #include <cmath>
@@ -82,6 +84,15 @@ struct DeviceGuard {
 };
 
 uint64_t round_up(uint64_t x, uint64_t a) { return (x + a - 1) / a * a; }
+
+// An NVTX range over one entry point, so a profiler's timeline shows the
+// library's calls (a no-op unless a tool is attached).
+struct Range {
+    explicit Range(const char* name) { nvtxRangePushA(name); }
+    ~Range() { nvtxRangePop(); }
+    Range(const Range&) = delete;
+    Range& operator=(const Range&) = delete;
+};
 
 // Polls an event until it completes or timeout_ms passes.
 lc_status wait_event(cudaEvent_t ev, int timeout_ms, const char* what) {
@@ -762,6 +773,7 @@ bool step_open(const lc_ctx* ctx) {
 }  // namespace
 
 extern "C" lc_status lc_measure(lc_ctx* ctx, int64_t step) {
+    Range range("lc_measure");
     g_err.clear();
     if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_measure: ctx is NULL");
     if (ctx->state == kNew) return fail(LC_ERR_STATE, "lc_measure: no layout registered");
@@ -842,6 +854,7 @@ extern "C" lc_status lc_register_optimizer(lc_ctx* ctx, const lc_optim_segment* 
 }
 
 extern "C" lc_status lc_adamw_step_measure(lc_ctx* ctx, int64_t step, const lc_adamw_hparams* hp) {
+    Range range("lc_adamw_step_measure");
     g_err.clear();
     if (!ctx || !hp) return fail(LC_ERR_INVALID_ARG, "lc_adamw_step_measure: NULL argument");
     if (!ctx->d_opt) return fail(LC_ERR_STATE, "lc_adamw_step_measure: no optimizer registered");
@@ -902,6 +915,7 @@ extern "C" lc_status lc_set_layer_sums_buffer(lc_ctx* ctx, double* sums_dev) {
 
 extern "C" lc_status lc_select(lc_ctx* ctx, double tau, int32_t max_staleness, uint8_t* mask_out,
                                double* u_out, uint64_t* bytes_out) {
+    Range range("lc_select");
     g_err.clear();
     if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_select: ctx is NULL");
     if (ctx->state != kMeasured) return fail(LC_ERR_STATE, "lc_select: call lc_measure first");
@@ -995,6 +1009,7 @@ lc_status ensure_staging(lc_ctx* ctx) {
 }  // namespace
 
 extern "C" lc_status lc_pack_device(lc_ctx* ctx, void* dst, uint64_t dst_capacity) {
+    Range range("lc_pack_device");
     g_err.clear();
     if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_pack_device: ctx is NULL");
     if (ctx->state != kSelected) return fail(LC_ERR_STATE, "lc_pack_device: call lc_select first");
@@ -1015,6 +1030,7 @@ extern "C" lc_status lc_pack_device(lc_ctx* ctx, void* dst, uint64_t dst_capacit
 }
 
 extern "C" lc_status lc_pack_async(lc_ctx* ctx, lc_store* st) {
+    Range range("lc_pack_async");
     g_err.clear();
     if (!ctx || !st) return fail(LC_ERR_INVALID_ARG, "lc_pack_async: NULL argument");
     if (ctx->state != kSelected) return fail(LC_ERR_STATE, "lc_pack_async: call lc_select first");
@@ -1117,6 +1133,7 @@ extern "C" lc_status lc_pack_async(lc_ctx* ctx, lc_store* st) {
 }
 
 extern "C" lc_status lc_commit_snapshot(lc_ctx* ctx) {
+    Range range("lc_commit_snapshot");
     g_err.clear();
     if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_commit_snapshot: ctx is NULL");
     if (ctx->state == kSelected && ctx->hdr.n_selected == 0) {
@@ -1135,6 +1152,7 @@ extern "C" lc_status lc_commit_snapshot(lc_ctx* ctx) {
 }
 
 extern "C" lc_status lc_wait_durable(lc_ctx* ctx, int64_t step, int32_t timeout_ms) {
+    Range range("lc_wait_durable");
     g_err.clear();
     if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_wait_durable: ctx is NULL");
     const int tmo = timeout_ms > 0 ? timeout_ms : ctx->cfg.timeout_ms;
@@ -1224,6 +1242,7 @@ lc_status enqueue_step(lc_ctx* ctx, cudaStream_t s, int64_t step, bool step_from
 
 extern "C" lc_status lc_step_async(lc_ctx* ctx, int64_t step, double tau, int32_t max_staleness,
                                    void* dst, uint64_t dst_capacity) {
+    Range range("lc_step_async");
     g_err.clear();
     if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_step_async: ctx is NULL");
     if (ctx->state == kNew) return fail(LC_ERR_STATE, "lc_step_async: no layout registered");
@@ -1253,6 +1272,7 @@ extern "C" lc_status lc_step_async(lc_ctx* ctx, int64_t step, double tau, int32_
 
 extern "C" lc_status lc_step_wait(lc_ctx* ctx, int64_t step, int32_t timeout_ms, uint8_t* mask_out,
                                   double* u_out, uint64_t* bytes_out) {
+    Range range("lc_step_wait");
     g_err.clear();
     if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_step_wait: ctx is NULL");
     lc_ctx::AsyncSlot* sl = nullptr;
@@ -1288,6 +1308,7 @@ extern "C" lc_status lc_step_wait(lc_ctx* ctx, int64_t step, int32_t timeout_ms,
 
 extern "C" lc_status lc_step_graph_create(lc_ctx* ctx, double tau, int32_t max_staleness, void* dst,
                                           uint64_t dst_capacity) {
+    Range range("lc_step_graph_create");
     g_err.clear();
     if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_step_graph_create: ctx is NULL");
     if (ctx->state == kNew) return fail(LC_ERR_STATE, "lc_step_graph_create: no layout registered");
@@ -1338,6 +1359,7 @@ extern "C" lc_status lc_step_graph_create(lc_ctx* ctx, double tau, int32_t max_s
 }
 
 extern "C" lc_status lc_step_graph_launch(lc_ctx* ctx, int64_t* step_out) {
+    Range range("lc_step_graph_launch");
     g_err.clear();
     if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_step_graph_launch: ctx is NULL");
     if (!ctx->graph_exec) return fail(LC_ERR_STATE, "lc_step_graph_launch: no graph (lc_step_graph_create)");
@@ -1365,6 +1387,7 @@ extern "C" lc_status lc_step_graph_launch(lc_ctx* ctx, int64_t* step_out) {
 // restore (§3.5, Eq. 8)
 // ---------------------------------------------------------------------------
 extern "C" lc_status lc_restore(lc_ctx* ctx, lc_store* st, int64_t t_fail, int64_t* layer_steps_out) {
+    Range range("lc_restore");
     g_err.clear();
     if (!ctx || !st) return fail(LC_ERR_INVALID_ARG, "lc_restore: NULL argument");
     if (ctx->state == kNew) return fail(LC_ERR_STATE, "lc_restore: no layout registered");
