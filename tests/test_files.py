@@ -156,3 +156,38 @@ def test_record_beyond_the_block_file_is_not_intact(tmp_path, P):
     got, _, _, torn = P.manifest_read(d, verify_blocks=True)
     assert not torn and len(got) == len(recs)
     assert [g["intact"] for g in got] == [1] * (len(recs) - 1) + [0]
+
+
+def test_pick_matches_composite_rule_and_replay():
+    """The record pick of recovery (§3.5, Eq. 8) against two other forms of
+    the same rule.  The first is the C oracle's composite pick over the same
+    versions, where an intact record of the right size and layout counts as
+    durable.  The second is a replay that applies the valid records at or
+    before t_fail in step order, record order breaking ties: each layer ends
+    on its pick.  Random logs with ties, out-of-range layers, wrong sizes,
+    foreign layouts and damaged blocks."""
+    from oracle import oracle as O
+    rng = np.random.default_rng(7)
+    layer_bytes = [4096, 768, 12288, 256, 512]
+    nl = len(layer_bytes)
+    lay = F.layout_crc(layer_bytes)
+    for _ in range(300):
+        recs = []
+        for _ in range(int(rng.integers(0, 40))):
+            l = int(rng.integers(-1, nl + 1))
+            in_range = 0 <= l < nl
+            recs.append(dict(layer=l, step=int(rng.integers(0, 8)), offset=0,
+                             bytes=layer_bytes[l] if in_range and rng.random() < 0.9 else 100,
+                             block_crc=0, layout_crc=lay if rng.random() < 0.95 else lay ^ 1,
+                             intact=bool(rng.random() < 0.85)))
+        t_fail = int(rng.integers(-1, 9))
+        pk = F.pick(recs, layer_bytes, t_fail)
+        valid = [bool(r["intact"]) and 0 <= r["layer"] < nl and r["bytes"] == layer_bytes[r["layer"]]
+                 and r["layout_crc"] == lay for r in recs]
+        cp = O.composite_pick([r["layer"] for r in recs], [r["step"] for r in recs], valid, nl, t_fail)
+        assert list(pk) == cp.tolist()
+        state = [-1] * nl
+        for i in sorted(range(len(recs)), key=lambda i: (recs[i]["step"], i)):
+            if valid[i] and recs[i]["step"] <= t_fail:
+                state[recs[i]["layer"]] = i
+        assert list(pk) == state

@@ -116,3 +116,90 @@ def test_genuine_oracle_passes_the_same_runner():
     r = subprocess.run([sys.executable, "-c", RUNNER, ROOT, build_oracle(), *names],
                        capture_output=True, text=True, timeout=600)
     assert r.returncode == 0, r.stdout + r.stderr
+
+
+# ----------------------------------------------------------------------------
+# the file-tier oracle (oracle/files.py): the same idea for its Python form
+# ----------------------------------------------------------------------------
+FILES_SRC = os.path.join(ROOT, "oracle", "files.py")
+
+FILES_MUTATIONS = [
+    ("crc-polynomial-term-dropped", "(0, 6, 8, 9, 10, 11, 13, 14, 18, 19, 20, 22, 23, 25, 26, 27, 28)",
+     "(0, 6, 8, 9, 10, 11, 13, 14, 18, 19, 20, 22, 23, 25, 26, 27)", ["test_crc32c_check_value_and_forms"]),
+    ("crc-no-final-inversion", "reg = (reg >> 8) ^ t[(reg ^ byte) & 0xFF]\n    return reg ^ 0xFFFFFFFF",
+     "reg = (reg >> 8) ^ t[(reg ^ byte) & 0xFF]\n    return reg", ["test_crc32c_check_value_and_forms"]),
+    ("crc-table-index-drops-register", "t[(reg ^ byte) & 0xFF]", "t[byte & 0xFF]",
+     ["test_crc32c_check_value_and_forms"]),
+    ("pick-tie-keeps-first-record", 'r["step"] >= recs[best[l]]["step"]', 'r["step"] > recs[best[l]]["step"]',
+     ["test_pick_matches_composite_rule_and_replay"]),
+    ("pick-past-t_fail", 'r["step"] > t_fail', 'r["step"] > t_fail + 1',
+     ["test_pick_matches_composite_rule_and_replay"]),
+    ("pick-ignores-damage", ' or not r.get("intact", True)', "",
+     ["test_pick_matches_composite_rule_and_replay", "test_damaged_block_is_not_intact"]),
+    ("pick-ignores-block-size", 'r["bytes"] != layer_bytes[l] or ', "",
+     ["test_pick_matches_composite_rule_and_replay"]),
+    ("reader-skips-a-bad-record", "            break\n        layer, step",
+     "            off += REC\n            continue\n        layer, step", ["test_torn_tail_and_damaged_record_end_the_log"]),
+    ("record-offset-and-size-swapped", 'pack("<iqQQII", layer, step, offset, nbytes, block_crc, layout)',
+     'pack("<iqQQII", layer, step, nbytes, offset, block_crc, layout)',
+     ["test_manifest_read_matches_independent_writer"]),
+    ("verify-ignores-block-crc", 'len(blk) == r["bytes"] and crc_of(blk) == r["block_crc"]', 'len(blk) == r["bytes"]',
+     ["test_damaged_block_is_not_intact"]),
+]
+
+RUNNER_FILES = r"""
+import importlib.util, pathlib, sys, tempfile
+sys.path.insert(0, sys.argv[1])
+import oracle
+spec = importlib.util.spec_from_file_location("oracle.files", sys.argv[2])
+mod = importlib.util.module_from_spec(spec)
+sys.modules["oracle.files"] = mod
+spec.loader.exec_module(mod)
+oracle.files = mod
+from tests import test_files as T
+P = None
+failed = []
+for name in sys.argv[3:]:
+    fn = T.__dict__[name]
+    args = fn.__code__.co_varnames[:fn.__code__.co_argcount]
+    kw = {}
+    if "P" in args:
+        if P is None:
+            from paper_2609_27193_gb300 import build as B
+            B.build()
+            import paper_2609_27193_gb300 as P
+        kw["P"] = P
+    with tempfile.TemporaryDirectory() as d:
+        if "tmp_path" in args:
+            kw["tmp_path"] = pathlib.Path(d)
+        try:
+            fn(**kw)
+        except Exception:
+            failed.append(name)
+print("FAILED:" + ",".join(failed))
+sys.exit(3 if failed else 0)
+"""
+
+
+def _files_mutant(old, new, tmp):
+    text = open(FILES_SRC).read()
+    assert text.count(old) == 1, "mutation anchor must occur exactly once: %r" % old
+    path = os.path.join(tmp, "files.py")
+    open(path, "w").write(text.replace(old, new))
+    return path
+
+
+@pytest.mark.parametrize("name,old,new,tests", FILES_MUTATIONS, ids=[m[0] for m in FILES_MUTATIONS])
+def test_file_tier_pins_catch_planted_mistake(name, old, new, tests):
+    with tempfile.TemporaryDirectory() as tmp:
+        path = _files_mutant(old, new, tmp)
+        r = subprocess.run([sys.executable, "-c", RUNNER_FILES, ROOT, path, *tests],
+                           capture_output=True, text=True, timeout=600)
+    assert r.returncode != 0, "mutation %s passed every pin in %s\n%s%s" % (name, tests, r.stdout, r.stderr)
+
+
+def test_genuine_file_tier_oracle_passes_the_same_runner():
+    names = sorted({t for m in FILES_MUTATIONS for t in m[3]})
+    r = subprocess.run([sys.executable, "-c", RUNNER_FILES, ROOT, FILES_SRC, *names],
+                       capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0, r.stdout + r.stderr
