@@ -73,11 +73,12 @@ typedef enum { LC_DRIFT_SNAPSHOT = 0, LC_DRIFT_ACCUMULATE = 1 } lc_drift_mode;
 
 /* How the kernels move bytes (the results are the same either way).
  * LC_COPY_BULK   : the bulk-copy engine (cp.async.bulk through shared-memory
- *                  rings, one load-issuing thread per SM) whenever every
+ *                  rings, one load-issuing thread per CTA) whenever every
  *                  address involved is device memory: the pack, commit and
  *                  restore copies (segments, staging ring and destination),
- *                  and in LC_DRIFT_SNAPSHOT mode the measure's reads of W and
- *                  R.  Otherwise as LC_COPY_THREADS (default).
+ *                  the measure's reads of W and R (and its R <- W in
+ *                  LC_DRIFT_ACCUMULATE mode), and the fused AdamW step.
+ *                  Otherwise as LC_COPY_THREADS (default).
  * LC_COPY_THREADS: every thread loads (and stores) 16-byte vectors. */
 typedef enum { LC_COPY_BULK = 0, LC_COPY_THREADS = 1 } lc_copy_engine;
 
