@@ -88,8 +88,10 @@ typedef enum { LC_COPY_BULK = 0, LC_COPY_THREADS = 1 } lc_copy_engine;
  * context's fault word and returns without finishing its work, and from
  * then on lc_select, lc_wait_durable, lc_step_wait and lc_restore fail with
  * LC_ERR_TIMEOUT.
+ * A launch of several waves of CTAs gives up wave after wave.
  * LC_DEBUG_BULK_STALL   : the pack / commit / restore copy kernel.
- * LC_DEBUG_MEASURE_STALL: the bulk-load measure kernel. */
+ * LC_DEBUG_MEASURE_STALL: the bulk-load measure kernel and the bulk-load
+ *                         fused AdamW step (they share the work partition). */
 #define LC_DEBUG_BULK_STALL 1
 #define LC_DEBUG_MEASURE_STALL 2
 
