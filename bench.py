@@ -303,6 +303,13 @@ def cpu_baseline(workload, seconds, use_gpu):
                       % (steps, meta["nlayers"], meta["params"], workload, total_t)}
 
 
+def ref_workload_label(name):
+    """The workload as the device arm names it in its config line."""
+    from lc_workloads.configs import WORKLOADS
+    shape = WORKLOADS[name].shape()
+    return "%s (%s, %d layers, %d params)" % (name, shape.name, shape.nlayers, shape.numel)
+
+
 def reference_arm(args):
     rank, world, _ = dist_env()
     if rank != 0:
@@ -324,7 +331,8 @@ def reference_arm(args):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * sum(ts) / len(ts), "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": args.workload, "sample": "4 transformer blocks"},
+            "config": {"workload": ref_workload_label(args.workload), "tau": tau, "max_staleness": K,
+                       "sample": "4 transformer blocks per step", "parallelism": "dp1"},
             "cpu_baseline": {"value": value, "unit": "GB/s", "cores": 1, "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0,
