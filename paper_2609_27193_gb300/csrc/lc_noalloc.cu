@@ -1,4 +1,4 @@
-// lc_noalloc.cu -- lc_measure_noalloc: the per-layer sums of Eq. 1 for
+// lc_noalloc.cu -- lc_measure_noalloc: the per-layer sums of lc_measure for
 // callers that cannot allocate device memory.
 //
 // It launches the same measure kernel as lc_measure, but every table and
@@ -7,9 +7,11 @@
 // LC_NOALLOC_SCRATCH_BYTES.  Host code never uses the array's name as an
 // address: at set-up, once per device and with that device current, the
 // array's device address is looked up with cudaGetSymbolAddress and cached.
-// The tables are built on the host in a fixed-size thread-local buffer and
-// copied into the array on the caller's stream; the completion counter
-// travels in that copy as zero.  No cudaMalloc, cudaFree or other
+// The tables are built on the host and reach the array as the kernel
+// parameters of small upload kernels launched on the caller's stream ahead
+// of the measure, so the driver copies them when each upload is launched and
+// nothing reads host memory once the call has returned.  The completion
+// counter travels in the upload as zero.  No cudaMalloc, cudaFree or other
 // allocating routine is called.
 #include "layercheck.h"
 #include "lc_internal.cuh"
@@ -30,15 +32,30 @@ constexpr int kMaxDevices = 64;
 
 constexpr size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
 
-// Scratch layout: tables first (uploaded every call), then kernel scratch.
-constexpr size_t kOffSegs = 0;
-constexpr size_t kOffCtaVec = al256(kOffSegs + sizeof(SegDev) * kMaxSeg);
-constexpr size_t kOffCtaSeg = al256(kOffCtaVec + sizeof(int64_t) * (kMaxCtas + 1));
-constexpr size_t kOffCtaSlot = al256(kOffCtaSeg + sizeof(int32_t) * kMaxCtas);
-constexpr size_t kOffSegSlot = al256(kOffCtaSlot + sizeof(int32_t) * kMaxCtas);
-constexpr size_t kOffLayerSeg = al256(kOffSegSlot + sizeof(int32_t) * (kMaxSeg + 1));
-constexpr size_t kOffTicket = al256(kOffLayerSeg + sizeof(int32_t) * (kMaxLayers + 1));
-constexpr size_t kTableBytes = al256(kOffTicket + sizeof(unsigned int));
+constexpr size_t al16(size_t x) { return (x + 15) & ~size_t(15); }
+
+// Where each table of one call sits in the array: the tables are packed
+// back to back (16-byte aligned) for the call's sizes, so the upload moves
+// only the bytes the measure will read.
+struct TableLayout {
+    size_t segs, cta_vec, cta_seg, cta_slot, seg_slot, layer_seg, ticket, bytes;
+};
+
+constexpr TableLayout table_layout(size_t nseg, size_t nlayers, size_t G) {
+    TableLayout t{};
+    t.segs = 0;
+    t.cta_vec = al16(t.segs + sizeof(SegDev) * nseg);
+    t.cta_seg = al16(t.cta_vec + sizeof(int64_t) * (G + 1));
+    t.cta_slot = al16(t.cta_seg + sizeof(int32_t) * G);
+    t.seg_slot = al16(t.cta_slot + sizeof(int32_t) * G);
+    t.layer_seg = al16(t.seg_slot + sizeof(int32_t) * (nseg + 1));
+    t.ticket = al16(t.layer_seg + sizeof(int32_t) * (nlayers + 1));
+    t.bytes = al16(t.ticket + sizeof(unsigned int));
+    return t;
+}
+
+// Scratch layout: the tables (at most kTableBytes), then the kernel scratch.
+constexpr size_t kTableBytes = al256(table_layout(kMaxSeg, kMaxLayers, kMaxCtas).bytes);
 constexpr size_t kOffPartials = kTableBytes;
 constexpr size_t kOffSegSums = al256(kOffPartials + sizeof(double2) * (kMaxCtas + kMaxSeg));
 constexpr size_t kScratchUsed = al256(kOffSegSums + sizeof(double) * 2 * kMaxSeg);
@@ -51,6 +68,27 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[LC_NOALLOC_SCRA
 
 namespace {
 
+// One upload: `nbytes` (a multiple of 16) of the table image, to be written
+// at byte `dst_off` of the scratch array.  Passed by value, so the launch
+// itself carries the bytes.
+constexpr int kUploadVecs = 1024;   // 16 KB of payload per launch
+struct UploadChunk {
+    uint32_t dst_off;
+    uint32_t nbytes;
+    uint4 data[kUploadVecs];
+};
+static_assert(sizeof(UploadChunk) <= 32000, "kernel parameters are limited to 32764 bytes");
+
+__global__ void __launch_bounds__(256) noalloc_upload_kernel(const __grid_constant__ UploadChunk c) {
+    uint4* dst = reinterpret_cast<uint4*>(g_noalloc_scratch + c.dst_off);
+    const uint32_t nv = c.nbytes / 16;
+    for (uint32_t i = threadIdx.x; i < nv; i += blockDim.x) dst[i] = c.data[i];
+}
+
+}  // namespace
+
+namespace {
+
 struct DeviceScratch {
     bool ready = false;
     unsigned char* addr = nullptr;   // device address of g_noalloc_scratch
@@ -59,8 +97,11 @@ struct DeviceScratch {
 DeviceScratch g_scratch[kMaxDevices];
 std::mutex g_scratch_mu;
 
-// Table image built on the host; one per host thread, no heap.
-thread_local unsigned char t_image[kTableBytes];
+// Table image built on the host; one per host thread, no heap.  The upload
+// launches copy it into their parameters, so it may be rebuilt as soon as
+// the call returns.
+thread_local unsigned char t_image[kTableBytes] __attribute__((aligned(16)));
+thread_local UploadChunk t_chunk;
 
 lc_status err(lc_status st, const char* fmt, ...) __attribute__((format(printf, 2, 3)));
 lc_status err(lc_status st, const char* fmt, ...) {
@@ -164,6 +205,8 @@ extern "C" lc_status lc_measure_noalloc(int device, void* cuda_stream, const lc_
             return err(LC_ERR_INVALID_ARG, "lc_measure_noalloc: segment %d has unknown dtype", i);
         if (s.numel <= 0 || !s.w || !s.snap)
             return err(LC_ERR_INVALID_ARG, "lc_measure_noalloc: segment %d needs numel > 0, w and snap", i);
+        if (s.snap == s.w)
+            return err(LC_ERR_INVALID_ARG, "lc_measure_noalloc: segment %d: snap must not alias w", i);
         const uintptr_t esz = s.w_dtype == LC_BF16 ? 2 : 4;
         if ((reinterpret_cast<uintptr_t>(s.w) % esz) || (reinterpret_cast<uintptr_t>(s.snap) % esz))
             return err(LC_ERR_INVALID_ARG, "lc_measure_noalloc: segment %d not element-aligned", i);
@@ -182,7 +225,9 @@ extern "C" lc_status lc_measure_noalloc(int device, void* cuda_stream, const lc_
     if (st != LC_OK) return st;
 
     std::memset(t_image, 0, sizeof t_image);
-    SegDev* sd = reinterpret_cast<SegDev*>(t_image + kOffSegs);
+    // the segment table sits at offset 0 whatever the grid; the rest of the
+    // layout depends on the grid, known once the work space is measured
+    SegDev* sd = reinterpret_cast<SegDev*>(t_image);
     int32_t fill[kMaxLayers];
     std::memcpy(fill, layer_begin, sizeof(int32_t) * nlayers);
     for (int32_t i = 0; i < nseg; ++i) {
@@ -204,15 +249,16 @@ extern "C" lc_status lc_measure_noalloc(int device, void* cuda_stream, const lc_
         sd[i].vec_begin = V;
         V += sd[i].nvec;
     }
-    const int64_t ngran_all = (V + LC_MEASURE_ALIGN_VECS - 1) / LC_MEASURE_ALIGN_VECS;
-    const int64_t G = ngran_all < ds.max_grid ? ngran_all : ds.max_grid;
-    int64_t* cta_vec = reinterpret_cast<int64_t*>(t_image + kOffCtaVec);
-    int32_t* cta_seg = reinterpret_cast<int32_t*>(t_image + kOffCtaSeg);
-    int32_t* cta_slot = reinterpret_cast<int32_t*>(t_image + kOffCtaSlot);
-    int32_t* seg_slot = reinterpret_cast<int32_t*>(t_image + kOffSegSlot);
-    int32_t* layer_seg = reinterpret_cast<int32_t*>(t_image + kOffLayerSeg);
-    for (int32_t i = 0; i <= nseg; ++i) seg_slot[i] = -1;
     const int64_t ngran = (V + LC_MEASURE_ALIGN_VECS - 1) / LC_MEASURE_ALIGN_VECS;
+    const int64_t G = ngran < ds.max_grid ? ngran : ds.max_grid;
+    const TableLayout L = table_layout(size_t(nseg), size_t(nlayers), size_t(G));
+    if (L.bytes > kTableBytes) return err(LC_ERR_CUDA, "lc_measure_noalloc: internal table overflow");
+    int64_t* cta_vec = reinterpret_cast<int64_t*>(t_image + L.cta_vec);
+    int32_t* cta_seg = reinterpret_cast<int32_t*>(t_image + L.cta_seg);
+    int32_t* cta_slot = reinterpret_cast<int32_t*>(t_image + L.cta_slot);
+    int32_t* seg_slot = reinterpret_cast<int32_t*>(t_image + L.seg_slot);
+    int32_t* layer_seg = reinterpret_cast<int32_t*>(t_image + L.layer_seg);
+    for (int32_t i = 0; i <= nseg; ++i) seg_slot[i] = -1;
     for (int64_t b = 0; b <= G; ++b) {
         const int64_t v = ngran * b / G * LC_MEASURE_ALIGN_VECS;
         cta_vec[b] = v < V ? v : V;
@@ -235,26 +281,33 @@ extern "C" lc_status lc_measure_noalloc(int device, void* cuda_stream, const lc_
     if (slot > kMaxCtas + kMaxSeg) return err(LC_ERR_CUDA, "lc_measure_noalloc: internal slot overflow");
 
     cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
-    // tables and a zero completion counter into the scratch array, stream-ordered
-    cudaError_t e = cudaMemcpyAsync(ds.addr, t_image, kTableBytes, cudaMemcpyHostToDevice, stream);
-    if (e != cudaSuccess) {
-        cudaGetLastError();
-        return err(LC_ERR_CUDA, "lc_measure_noalloc: table upload failed: %s", cudaGetErrorString(e));
+    // the tables and a zero completion counter into the scratch array,
+    // stream-ordered before the measure; each launch carries its bytes
+    cudaGetLastError();
+    for (size_t off = 0; off < L.bytes; off += sizeof t_chunk.data) {
+        const size_t n = L.bytes - off < sizeof t_chunk.data ? L.bytes - off : sizeof t_chunk.data;
+        t_chunk.dst_off = uint32_t(off);
+        t_chunk.nbytes = uint32_t(n);
+        std::memcpy(t_chunk.data, t_image + off, n);
+        noalloc_upload_kernel<<<1, 256, 0, stream>>>(t_chunk);
+        const cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess)
+            return err(LC_ERR_CUDA, "lc_measure_noalloc: table upload failed: %s", cudaGetErrorString(e));
     }
     MeasureParams p{};
-    p.segs = reinterpret_cast<const SegDev*>(ds.addr + kOffSegs);
-    p.cta_vec_begin = reinterpret_cast<const int64_t*>(ds.addr + kOffCtaVec);
-    p.cta_seg0 = reinterpret_cast<const int32_t*>(ds.addr + kOffCtaSeg);
-    p.cta_slot0 = reinterpret_cast<const int32_t*>(ds.addr + kOffCtaSlot);
-    p.seg_slot_begin = reinterpret_cast<const int32_t*>(ds.addr + kOffSegSlot);
-    p.layer_seg_begin = reinterpret_cast<const int32_t*>(ds.addr + kOffLayerSeg);
+    p.segs = reinterpret_cast<const SegDev*>(ds.addr + L.segs);
+    p.cta_vec_begin = reinterpret_cast<const int64_t*>(ds.addr + L.cta_vec);
+    p.cta_seg0 = reinterpret_cast<const int32_t*>(ds.addr + L.cta_seg);
+    p.cta_slot0 = reinterpret_cast<const int32_t*>(ds.addr + L.cta_slot);
+    p.seg_slot_begin = reinterpret_cast<const int32_t*>(ds.addr + L.seg_slot);
+    p.layer_seg_begin = reinterpret_cast<const int32_t*>(ds.addr + L.layer_seg);
     p.partials = reinterpret_cast<double2*>(ds.addr + kOffPartials);
     p.seg_sums = reinterpret_cast<double*>(ds.addr + kOffSegSums);
     p.sums = sums_out;
-    p.ticket = reinterpret_cast<unsigned int*>(ds.addr + kOffTicket);
+    p.ticket = reinterpret_cast<unsigned int*>(ds.addr + L.ticket);
     p.nseg = nseg;
     p.nlayers = nlayers;
-    e = launch_measure(p, int(G), false, stream);
+    const cudaError_t e = launch_measure(p, int(G), false, stream);
     if (e != cudaSuccess) {
         cudaGetLastError();
         return err(LC_ERR_CUDA, "lc_measure_noalloc: launch failed: %s", cudaGetErrorString(e));
