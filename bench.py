@@ -68,6 +68,13 @@ def parse_args():
                     help="also append every e2e step's persisted versions to the checkpoint "
                          "directory DIR (fsync'd), then time the metadata-driven recovery from it "
                          "(lc_store_load_dir + lc_restore); DIR is removed afterwards")
+    ap.add_argument("--copy-trace", default=None, metavar="FILE",
+                    help="write every span of the library's copy trace in the e2e loop and the "
+                         "restore (per staging chunk: kind, step, bytes, start/end ms) to FILE "
+                         "as JSON lines")
+    ap.add_argument("--no-dma-check", action="store_true",
+                    help="do not run lc_store_check_dma on the e2e store (by default the pinned "
+                         "regions the GPU copies into at under half the median rate are kept out of use)")
     ap.add_argument("--lean", action="store_true",
                     help="no fp32 master weights in the generator (small case for kernel captures)")
     return ap.parse_args()
@@ -375,7 +382,7 @@ def files_recovery(P, lc, path, t_fail, written, write_s):
             "oldest_version_step": int(min(steps)), "t_fail": int(t_fail)}
 
 
-def restore_leg(torch, dev, P, lc, store, t, tau, full):
+def restore_leg(torch, dev, P, lc, store, t, tau, full, trace_file=None):
     """§3.5 restore timed on its own: one step that persists every layer
     (S_max = 0) into the cleared store, then lc_restore of that composite
     (host -> device copies through the staging ring, scatter into W, m, v
@@ -387,9 +394,16 @@ def restore_leg(torch, dev, P, lc, store, t, tau, full):
     lc.commit_snapshot()
     lc.wait_durable(t)
     torch.cuda.synchronize()
+    lc.trace_copies(True)
     t0 = time.perf_counter()
     lc.restore(store, t)
     t1 = time.perf_counter()
+    spans, _ = lc.copy_trace()
+    lc.trace_copies(False)
+    if trace_file:
+        with open(trace_file, "a") as fh:
+            for x in spans:
+                fh.write(json.dumps(dict(x, loop_step=t)) + "\n")
     h = torch.empty(4 << 30, dtype=torch.uint8, pin_memory=True)
     d = torch.empty(4 << 30, dtype=torch.uint8, device=dev)
     best = 0.0
@@ -400,7 +414,43 @@ def restore_leg(torch, dev, P, lc, store, t, tau, full):
         torch.cuda.synchronize()
         best = max(best, h.numel() / (time.perf_counter() - a) / 1e9)
     del h, d
-    return {"bytes": int(full), "s": t1 - t0, "GBps": full / (t1 - t0) / 1e9, "h2d_link_GBps_measured": best}
+    return {"bytes": int(full), "s": t1 - t0, "GBps": full / (t1 - t0) / 1e9, "h2d_link_GBps_measured": best,
+            "h2d_trace": span_summary(spans, "h2d"), "scatter_trace": span_summary(spans, "scatter")}
+
+
+def span_summary(spans, kind):
+    """Chunk spans of one kind from the library's copy trace: bytes, the
+    time the stream spent on them (busy), the window from the first start to
+    the last end, and the chunks' own rates."""
+    sp = [x for x in spans if x["kind"] == kind and math.isfinite(x["start_ms"]) and x["end_ms"] > x["start_ms"]]
+    if not sp:
+        return None
+    busy = sum(x["end_ms"] - x["start_ms"] for x in sp)
+    window = max(x["end_ms"] for x in sp) - min(x["start_ms"] for x in sp)
+    nbytes = sum(x["bytes"] for x in sp)
+    rates = sorted(x["bytes"] / ((x["end_ms"] - x["start_ms"]) / 1e3) / 1e9 for x in sp)
+    pick = lambda q: rates[min(len(rates) - 1, int(q * len(rates)))]
+    return {"chunks": len(sp), "bytes": int(nbytes), "busy_ms": busy, "window_ms": window,
+            "idle_ms": max(0.0, window - busy), "busy_GBps": nbytes / (busy / 1e3) / 1e9,
+            "window_GBps": nbytes / (window / 1e3) / 1e9 if window > 0 else None,
+            "chunk_GBps_min": rates[0], "chunk_GBps_p10": pick(0.1), "chunk_GBps_p50": pick(0.5),
+            "chunk_GBps_p90": pick(0.9), "chunk_GBps_max": rates[-1]}
+
+
+def merge_span_summaries(items):
+    """Totals over several steps' summaries of one kind."""
+    items = [x for x in items if x]
+    if not items:
+        return None
+    busy = sum(x["busy_ms"] for x in items)
+    window = sum(x["window_ms"] for x in items)
+    nbytes = sum(x["bytes"] for x in items)
+    return {"steps": len(items), "chunks": sum(x["chunks"] for x in items), "bytes": int(nbytes),
+            "busy_ms": busy, "window_ms": window, "idle_frac": max(0.0, window - busy) / window if window else None,
+            "busy_GBps": nbytes / (busy / 1e3) / 1e9, "window_GBps": nbytes / (window / 1e3) / 1e9,
+            "chunk_GBps_p10_min": min(x["chunk_GBps_p10"] for x in items),
+            "chunk_GBps_p50_median": statistics.median(x["chunk_GBps_p50"] for x in items),
+            "chunk_GBps_p90_max": max(x["chunk_GBps_p90"] for x in items)}
 
 
 def d2h_link_probe(torch, dev, nbytes=4 << 30):
@@ -695,14 +745,33 @@ def run_ours(args):
                         avail = int(line.split()[1]) * 1024
         except OSError:
             pass
-        cap = full if avail == 0 else min(full, int(avail * 0.6))
+        dma_check = None
         if graph:
             # the replayed pack writes straight into pinned host memory
+            cap = full if avail == 0 else min(full, int(avail * 0.6))
             store = None
             hostdst = torch.empty(cap, dtype=torch.uint8, pin_memory=True)
             lc.step_graph_create(tau, K, hostdst)
         else:
+            # a quarter of the full state as headroom for regions the DMA
+            # check keeps out of use (pinned pages the GPU reaches slowly)
+            cap = int(full * 1.25) if avail == 0 else min(int(full * 1.25), int(avail * 0.6))
             store = P.Store(lc, capacity_bytes=cap)
+            if not args.no_dma_check:
+                region = 256 << 20
+                tchk = time.perf_counter()
+                rates, excluded = store.check_dma(lc, region_bytes=region, min_fraction=0.5, passes=6)
+                srt = np.sort(rates)
+                dma_check = {"region_bytes": region, "regions": int(rates.size), "passes": 6, "min_fraction": 0.5,
+                             "excluded_bytes": int(excluded), "excluded_regions": int(excluded // region),
+                             "worst_pass_GBps_median": float(srt[srt.size // 2]),
+                             "worst_pass_GBps_p10": float(srt[srt.size // 10]), "worst_pass_GBps_min": float(srt[0]),
+                             "capacity": int(cap), "s": time.perf_counter() - tchk}
+                if cap - excluded < full:
+                    # too little room left for a full step: keep every region
+                    store.close()
+                    store = P.Store(lc, capacity_bytes=cap)
+                    dma_check["dropped"] = "exclusions would leave less than the full state; none applied"
         link = d2h_link_probe(torch, dev)
         e_recs, e_bytes = [], []
         f_bytes, f_s = 0, 0.0
@@ -715,9 +784,20 @@ def run_ours(args):
             if need + (8 << 30) > free:
                 files_note = ("skipped: about %.0f GB would be written, %.0f GB free on %s"
                               % (need / 1e9, free / 1e9, args.files))
+        traces = []
         for i in range(max(1, args.warmup) + args.steps):
             t += 1
+            if store is not None:
+                lc.trace_copies(True)
             r = step(t, "store", store)
+            if store is not None:
+                spans, _ = lc.copy_trace()
+                if args.copy_trace:
+                    with open(args.copy_trace, "a") as fh:
+                        for x in spans:
+                            fh.write(json.dumps(dict(x, loop_step=t)) + "\n")
+                r["d2h_trace"] = span_summary(spans, "d2h")
+                r["gather_trace"] = span_summary(spans, "gather")
             if store is not None and args.files and files_note is None:
                 f0 = time.perf_counter()
                 f_bytes += store.persist_dir(args.files, sync=True)
@@ -727,6 +807,8 @@ def run_ours(args):
             if i >= max(1, args.warmup):
                 e_recs.append(r)
                 e_bytes.append(mbytes + pack_bytes(r["mask"], payload, wbytes, fused_commit=pack_commit))
+        if store is not None:
+            lc.trace_copies(False)
         link_after = d2h_link_probe(torch, dev)
         e_s = sum(r["host_s"] for r in e_recs)
         d2h = statistics.mean(r["nbytes"] for r in e_recs)
@@ -739,16 +821,27 @@ def run_ours(args):
                # machine: the same copy has measured 50-193 GB/s minutes apart, so
                # the link is probed right before and right after the loop
                "d2h_link_GBps_measured": link,
+               "store_dma_check": dma_check,
                "d2h_link_GBps_after": link_after,
                "steps_d2h_ms": [round(1e3 * ((r["host_s"] - r["decision_s"]) if not graph else r["host_s"]), 3)
                                 for r in e_recs],
                "steps_d2h_bytes": [int(r["nbytes"]) for r in e_recs],
+               # the library's own per-chunk events: D2H spans on its copy
+               # stream (busy = copying, idle = waiting for a gathered chunk)
+               # and the gathers into the staging slots on the context stream
+               "d2h_trace": merge_span_summaries([r.get("d2h_trace") for r in e_recs]),
+               "gather_trace": merge_span_summaries([r.get("gather_trace") for r in e_recs]),
+               "steps_d2h_busy_GBps": [round(r["d2h_trace"]["busy_GBps"], 1) if r.get("d2h_trace") else None
+                                       for r in e_recs],
+               "steps_d2h_idle_ms": [round(r["d2h_trace"]["idle_ms"], 2) if r.get("d2h_trace") else None
+                                     for r in e_recs],
                "note": "weights, snapshot and moments are device-resident training state; the "
                        "step's only host traffic is the decision block and the persisted "
                        "layers copied into %s" % ("pinned host memory by the replayed graph's pack"
                                                   if graph else "the pinned store")}
         if store is not None and cap >= full:
-            e2e["restore"] = restore_leg(torch, dev, P, lc, store, t + 1, tau, full)
+            e2e["restore"] = restore_leg(torch, dev, P, lc, store, t + 1, tau, full,
+                                         trace_file=args.copy_trace)
             t += 1
         if store is not None:
             store.close()

@@ -88,7 +88,10 @@ typedef enum { LC_COPY_BULK = 0, LC_COPY_THREADS = 1 } lc_copy_engine;
  * context's fault word and returns without finishing its work, and from
  * then on lc_select, lc_wait_durable, lc_step_wait and lc_restore fail with
  * LC_ERR_TIMEOUT.
- * A launch of several waves of CTAs gives up wave after wave.
+ * Every CTA of the copy kernel reads a device-memory copy of the fault word
+ * before its first load and returns at once if it is set, so a copy launch
+ * of several waves of CTAs ends soon after its first wave gave up, and later
+ * copy launches of the context end at once.
  * LC_DEBUG_BULK_STALL   : the pack / commit / restore copy kernel.
  * LC_DEBUG_MEASURE_STALL: the bulk-load measure kernel and the bulk-load
  *                         fused AdamW step (they share the work partition). */
@@ -256,9 +259,11 @@ lc_status lc_pack_device(lc_ctx* ctx, void* dst, uint64_t dst_capacity);
  * pinned host memory (device->host copies on the library's copy stream).
  * Records one pending version per selected layer; they become durable in
  * lc_wait_durable (a step that persisted nothing is durable at once).
- * Asynchronous.  Errors: STATE (no select, or the store
- * still holds a pending version of a layer it would overwrite),
- * INVALID_ARG (store built for another layout), CAPACITY, CUDA. */
+ * Asynchronous, except that with a newest-only store it may wait for
+ * copies of this step to make room (see lc_store_create).  Errors: STATE (no
+ * select, or the store still holds a pending version of a layer it would
+ * overwrite; for a newest-only store, any pending version), INVALID_ARG
+ * (store built for another layout), CAPACITY, TIMEOUT, CUDA. */
 lc_status lc_pack_async(lc_ctx* ctx, lc_store* store);
 
 /* Snapshot mode: enqueues snap <- w for the layers persisted this step
@@ -366,12 +371,67 @@ lc_status lc_register_optimizer(lc_ctx* ctx, const lc_optim_segment* segs, int32
  * Errors: STATE (no optimizer registered, or a step is open), INVALID_ARG. */
 lc_status lc_adamw_step_measure(lc_ctx* ctx, int64_t step, const lc_adamw_hparams* hp);
 
+/* --- copy trace (measurement of the staged host copies) ---------------- */
+
+/* What a traced span timed.  lc_pack_async stages its stream through the
+ * device staging ring in chunks: for each chunk a GATHER span on the
+ * context's stream (the pack kernel into a staging slot) and a D2H span on
+ * the library's copy stream (the device->host copies of that slot into the
+ * store).  lc_restore does the reverse: an H2D span on the copy stream, then
+ * a SCATTER span on the context's stream. */
+#define LC_SPAN_GATHER 0
+#define LC_SPAN_D2H 1
+#define LC_SPAN_H2D 2
+#define LC_SPAN_SCATTER 3
+
+typedef struct {
+    int32_t kind;       /* LC_SPAN_*                                            */
+    int32_t chunk;      /* chunk index within its lc_pack_async / lc_restore    */
+    int64_t step;       /* the packed step, or t_fail of the restore            */
+    uint64_t bytes;     /* bytes of the packed stream the chunk covers          */
+    double start_ms;    /* ms after the first recorded span started (NaN if the */
+    double end_ms;      /* span could not be timed)                             */
+} lc_copy_span;
+
+/* Starts (enable != 0) or stops recording spans; either way the previous
+ * record is cleared.  A span's start event is recorded on its stream just
+ * before its work and its end event just after, so end - start is the work
+ * itself, and the gap between consecutive spans of one stream is time that
+ * stream spent waiting (for the other stream or for its own earlier work).
+ * Costs two CUDA events per span; at most 65536 spans are kept, later ones
+ * are counted as dropped.  Errors: INVALID_ARG. */
+lc_status lc_copy_trace_enable(lc_ctx* ctx, int32_t enable);
+
+/* Waits (bounded by the config's timeout_ms) for the recorded spans and
+ * copies up to `cap` of them, in record order, into `out` (host).  *n_out
+ * (nullable): spans recorded; *dropped_out (nullable): spans not kept.  Does
+ * not clear the record.  Errors: INVALID_ARG, TIMEOUT, CUDA. */
+lc_status lc_copy_trace_read(lc_ctx* ctx, lc_copy_span* out, int64_t cap, int64_t* n_out,
+                             int64_t* dropped_out);
+
 /* --- persisted-version store (pinned host memory) ---------------------- */
 
 /* Creates a store for the layout registered in ctx.
  * versions_per_layer = 0: an append-only log of every version in one
  *   pinned arena of capacity_bytes (every restore point stays available
  *   until lc_store_clear).
+ * versions_per_layer = 1: newest-only.  An arena of capacity_bytes holds
+ *   each layer's newest durable version.  Layers whose blocks have the same
+ *   size share a class of slots: the class's layers' slots, one spare, and
+ *   further spares as capacity_bytes allows (4096-byte aligned).  A new
+ *   version goes into a free slot of its class, and the layer's previous
+ *   version frees its slot only once the new one is durable, so a crash
+ *   during a copy still leaves the previous version.  Durability is per
+ *   layer: a version counts as durable as soon as its own copy has completed.
+ *   When a class has no free slot, lc_pack_async waits (host side, bounded by
+ *   timeout_ms) for the copy of the step's earliest layer of that class not
+ *   yet seen complete, whose previous version's slot then serves; so every
+ *   step fits, whatever it persists, in every layer's block plus one block of
+ *   each distinct size (the minimum capacity_bytes accepted).  The placement
+ *   is decided before anything is enqueued: LC_ERR_CAPACITY (possible only
+ *   after exclusions) leaves the store untouched.  lc_pack_async needs every
+ *   earlier version durable (lc_wait_durable).  Only the newest restore point
+ *   of each layer is available.
  * versions_per_layer = V >= 2: each layer owns V block slots and keeps its
  *   V newest versions; capacity_bytes is ignored.  Restore points older
  *   than a layer's oldest kept version are no longer available.
@@ -386,7 +446,47 @@ void lc_store_destroy(lc_store* store);
 lc_status lc_store_clear(lc_store* store);
 
 int64_t lc_store_num_versions(const lc_store* store);
+
+/* A store's arena and its use. */
+typedef struct {
+    const void* arena;         /* pinned host base address of the arena         */
+    uint64_t capacity;         /* arena bytes                                   */
+    uint64_t excluded_bytes;   /* bytes kept out of use (lc_store_exclude)      */
+    uint64_t used_bytes;       /* bytes held by versions, pending or durable    */
+    int32_t versions_per_layer;
+    int32_t reserved;
+} lc_store_info;
+
+/* Errors: INVALID_ARG (NULL). */
+lc_status lc_store_get_info(const lc_store* store, lc_store_info* out);
 lc_status lc_store_get_version(const lc_store* store, int64_t index, lc_version* out);
+
+/* Takes bytes [offset, offset + bytes) of the store's arena (widened to
+ * whole 4096-byte granules) out of use: no later version is placed there.
+ * Log and newest-only stores; the range must hold no version.  Excluded
+ * ranges stay excluded across lc_store_clear.  A log store places each layer
+ * block at the next offset whose block touches no excluded range.
+ * Errors: INVALID_ARG (ring store, range outside the arena), STATE (a
+ * version lies in the range). */
+lc_status lc_store_exclude(lc_store* store, uint64_t offset, uint64_t bytes);
+
+/* Pinned host memory is not uniform for the GPU: on a shared host some of
+ * its pages can take device copies at a small fraction of the link rate,
+ * and not all the time (measured here: a fixed set of a few GB of an 80 GB
+ * pinned arena copying at 15-60 GB/s in about half of the passes over it,
+ * the rest at 193 GB/s in every pass).  This times `passes` device->host
+ * copies into every region_bytes region of an empty log or newest-only
+ * store (from a device buffer on ctx's device) and excludes
+ * (lc_store_exclude) every region whose slowest pass ran below min_fraction
+ * times the median of the regions' fastest passes.  region_bytes: 0 (256
+ * MiB) or a multiple of 4096 in [1 MiB, 1 GiB]; passes: 0 (4) or 1..64.
+ * rates_out (host, nullable): each of the ceil(capacity / region_bytes)
+ * regions' slowest GB/s; excluded_out (nullable): bytes excluded.
+ * Overwrites the arena; blocks (bounded by ctx's timeout_ms).
+ * Errors: INVALID_ARG, STATE (the store holds versions), TIMEOUT, CUDA,
+ * OOM. */
+lc_status lc_store_check_dma(lc_store* store, lc_ctx* ctx, uint64_t region_bytes, int32_t passes,
+                             double min_fraction, double* rates_out, int64_t rates_cap, uint64_t* excluded_out);
 
 /* §3.5 reconstruction plan: pick_out[l] = index of the durable version of
  * layer l with the largest step <= t_fail (the newer record on a tie), or
@@ -469,16 +569,20 @@ lc_status lc_manifest_read(const char* dir, int32_t verify_blocks, lc_manifest_r
  * cudaMalloc once they are running: a framework that owns every byte of
  * the GPU through its own memory pool, a process whose device footprint is
  * fixed at start-up, or code where an allocation could synchronize the
- * device at a bad moment.  Such a caller can still get the per-layer sums of
- * Eq. 1 from this call without creating a context.
+ * device at a bad moment.  Such a caller can still get the per-layer sums
+ * that lc_measure computes from this call, without an lc_ctx.
  *
  * Computes, on `cuda_stream` of `device`, the same per-layer sums as
  * lc_measure: sums_out[3*l] = sum |W - R|, sums_out[3*l+1] = sum |R|,
  * sums_out[3*l+2] = element count of layer l, for the segments `segs` (host
- * array of nseg lc_segment, the layout rules of lc_register_layout; snap is
- * only read, exp_avg / exp_avg_sq are ignored).  sums_out: caller-owned
- * device memory of 3*nlayers fp64, 8-byte aligned.  Asynchronous; the host
- * array may be reused when the call returns.
+ * array of nseg lc_segment in any layer order, the layout rules of
+ * lc_register_layout: snap is required and must not alias w; it is only
+ * read, exp_avg / exp_avg_sq are ignored).  A layer's segments are summed in
+ * their order within `segs`.  sums_out: caller-owned device memory of
+ * 3*nlayers fp64, 8-byte aligned.  Asynchronous.  The segment table and the
+ * work partition travel to the device inside the call's own kernel
+ * launches, so the host array may be reused, and nothing on the host is
+ * read, once the call has returned.
  *
  * Memory: the call allocates nothing.  Its scratch (tables, partial sums,
  * completion counter) lives in one static device array of

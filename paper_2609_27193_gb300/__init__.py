@@ -286,6 +286,25 @@ class LayerCheck:
         check(self._lib.lc_layer_block_bytes(self._ctx, int(layer), C.byref(b)))
         return b.value
 
+    def trace_copies(self, enable=True):
+        """Start (or stop) timing the staged host copies of pack_async and
+        restore chunk by chunk; clears the previous record."""
+        check(self._lib.lc_copy_trace_enable(self._ctx, int(bool(enable))))
+
+    def copy_trace(self):
+        """The recorded spans as a list of dicts (kind, chunk, step, bytes,
+        start_ms, end_ms), in record order, and the number dropped."""
+        from ._abi import SPAN_NAMES, lc_copy_span
+        n = C.c_int64(0)
+        dropped = C.c_int64(0)
+        check(self._lib.lc_copy_trace_read(self._ctx, None, 0, C.byref(n), C.byref(dropped)))
+        arr = (lc_copy_span * max(1, n.value))()
+        check(self._lib.lc_copy_trace_read(self._ctx, arr, n.value, C.byref(n), C.byref(dropped)))
+        out = [dict(kind=SPAN_NAMES.get(arr[i].kind, arr[i].kind), chunk=arr[i].chunk, step=arr[i].step,
+                    bytes=arr[i].bytes, start_ms=arr[i].start_ms, end_ms=arr[i].end_ms)
+               for i in range(n.value)]
+        return out, dropped.value
+
     def counters(self):
         c = lc_counters()
         check(self._lib.lc_get_counters(self._ctx, C.byref(c)))
@@ -353,6 +372,35 @@ class Store:
             return np.zeros(0, np.uint8)
         buf = (C.c_uint8 * v["bytes"]).from_address(v["host_ptr"])
         return np.frombuffer(buf, dtype=np.uint8)
+
+    def info(self):
+        """Arena base address, capacity, excluded and used bytes."""
+        from ._abi import lc_store_info
+        i = lc_store_info()
+        check(self._lib.lc_store_get_info(self._h, C.byref(i)))
+        return dict(arena=i.arena, capacity=i.capacity, excluded_bytes=i.excluded_bytes,
+                    used_bytes=i.used_bytes, versions_per_layer=i.versions_per_layer)
+
+    @property
+    def capacity(self):
+        return self.info()["capacity"]
+
+    def exclude(self, offset, nbytes):
+        """Keep bytes [offset, offset + nbytes) of the arena out of use."""
+        check(self._lib.lc_store_exclude(self._h, int(offset), int(nbytes)))
+
+    def check_dma(self, lc, region_bytes=256 << 20, min_fraction=0.5, passes=4):
+        """Time `passes` device->host copies into every region of the (empty)
+        arena and exclude the regions whose slowest pass ran below
+        min_fraction x the median of the regions' fastest passes.  Returns
+        (each region's slowest GB/s as a numpy array, excluded bytes)."""
+        cap = int(self.capacity)
+        n = -(-cap // int(region_bytes))
+        rates = np.zeros(n, dtype=np.float64)
+        ex = C.c_uint64(0)
+        check(self._lib.lc_store_check_dma(self._h, lc.handle, int(region_bytes), int(passes),
+                                           float(min_fraction), rates.ctypes.data, n, C.byref(ex)))
+        return rates, ex.value
 
     def plan(self, t_fail):
         pick = np.zeros(self.nlayers, dtype=np.int64)

@@ -25,6 +25,8 @@ LC_DRIFT_SNAPSHOT, LC_DRIFT_ACCUMULATE = 0, 1
 LC_COPY_BULK, LC_COPY_THREADS = 0, 1
 LC_DEBUG_BULK_STALL = 1
 LC_DEBUG_MEASURE_STALL = 2
+LC_SPAN_GATHER, LC_SPAN_D2H, LC_SPAN_H2D, LC_SPAN_SCATTER = 0, 1, 2, 3
+SPAN_NAMES = {0: "gather", 1: "d2h", 2: "h2d", 3: "scatter"}
 
 
 class lc_segment(C.Structure):
@@ -74,6 +76,16 @@ class lc_manifest_record(C.Structure):
                 ("layout_crc", C.c_uint32)]
 
 
+class lc_store_info(C.Structure):
+    _fields_ = [("arena", C.c_void_p), ("capacity", C.c_uint64), ("excluded_bytes", C.c_uint64),
+                ("used_bytes", C.c_uint64), ("versions_per_layer", C.c_int32), ("reserved", C.c_int32)]
+
+
+class lc_copy_span(C.Structure):
+    _fields_ = [("kind", C.c_int32), ("chunk", C.c_int32), ("step", C.c_int64),
+                ("bytes", C.c_uint64), ("start_ms", C.c_double), ("end_ms", C.c_double)]
+
+
 ctx_p = C.c_void_p
 store_p = C.c_void_p
 P = C.POINTER
@@ -104,6 +116,10 @@ SIGNATURES = {
     "lc_store_num_versions": (C.c_int64, [store_p]),
     "lc_store_get_version": (C.c_int, [store_p, C.c_int64, P(lc_version)]),
     "lc_store_plan": (C.c_int, [store_p, C.c_int64, C.c_void_p]),
+    "lc_store_exclude": (C.c_int, [store_p, C.c_uint64, C.c_uint64]),
+    "lc_store_get_info": (C.c_int, [store_p, P(lc_store_info)]),
+    "lc_store_check_dma": (C.c_int, [store_p, ctx_p, C.c_uint64, C.c_int32, C.c_double, C.c_void_p,
+                                     C.c_int64, P(C.c_uint64)]),
     "lc_step_async": (C.c_int, [ctx_p, C.c_int64, C.c_double, C.c_int32, C.c_void_p, C.c_uint64]),
     "lc_step_wait": (C.c_int, [ctx_p, C.c_int64, C.c_int32, C.c_void_p, C.c_void_p, P(C.c_uint64)]),
     "lc_step_graph_create": (C.c_int, [ctx_p, C.c_double, C.c_int32, C.c_void_p, C.c_uint64]),
@@ -112,6 +128,8 @@ SIGNATURES = {
     "lc_adamw_step_measure": (C.c_int, [ctx_p, C.c_int64, P(lc_adamw_hparams)]),
     "lc_measure_noalloc": (C.c_int, [C.c_int, C.c_void_p, P(lc_segment), C.c_int32, C.c_int32,
                                      C.c_void_p]),
+    "lc_copy_trace_enable": (C.c_int, [ctx_p, C.c_int32]),
+    "lc_copy_trace_read": (C.c_int, [ctx_p, P(lc_copy_span), C.c_int64, P(C.c_int64), P(C.c_int64)]),
     "lc_crc32c": (C.c_uint32, [C.c_void_p, C.c_uint64, C.c_uint32]),
     "lc_store_persist_dir": (C.c_int, [store_p, C.c_char_p, C.c_int32, P(C.c_uint64)]),
     "lc_store_load_dir": (C.c_int, [ctx_p, C.c_char_p, C.c_int64, P(store_p), C.c_void_p]),

@@ -18,6 +18,8 @@
 #include <cstdio>
 #include <cstring>
 #include <exception>
+#include <iterator>
+#include <map>
 #include <mutex>
 #include <set>
 #include <string>
@@ -149,17 +151,98 @@ struct StoreVersion {
 
 struct lc_store {
     int32_t nlayers = 0;
-    int32_t per_layer = 0;                 // 0 = log
+    int32_t per_layer = 0;                 // 0 = log, 1 = newest-only, V >= 2 = ring
     uint64_t capacity = 0;
     uint8_t* arena = nullptr;
     uint64_t top = 0;                      // log mode
     std::vector<uint64_t> layer_bytes;
     std::vector<uint64_t> layer_base;      // ring mode
     std::vector<int64_t> layer_writes;     // ring mode: versions ever written
+    std::map<uint64_t, uint64_t> excluded; // ranges kept out of use (lc_store_exclude), disjoint
+    // newest-only mode: layers whose blocks have the same size share a class
+    // of slots (its layers' slots plus spares); a free slot list per class
+    std::vector<int32_t> layer_class;
+    std::vector<uint64_t> class_bytes;     // slot size (block size rounded to 4096)
+    std::vector<int32_t> class_layers;
+    std::vector<int32_t> class_slots;      // slots laid out in the arena
+    std::vector<std::vector<uint64_t>> class_free;
     std::vector<StoreVersion> versions;
     int64_t next_id = 0;
     std::vector<cudaEvent_t> inflight;     // copies still writing into the arena
 };
+
+namespace {
+
+// Blocks of a newest-only store start on this boundary.
+constexpr uint64_t kStoreGrain = 4096;
+
+// Log mode: the first offset >= `from` at which `len` bytes touch no
+// excluded range.
+uint64_t log_place(const lc_store* st, uint64_t from, uint64_t len) {
+    uint64_t at = from;
+    for (const auto& x : st->excluded) {
+        if (x.first + x.second <= at) continue;
+        if (at + len <= x.first) break;
+        at = x.first + x.second;
+    }
+    return at;
+}
+
+// Newest-only mode: lays the slots out in an empty store, skipping excluded
+// ranges -- classes largest first, each its layers' slots plus one spare,
+// then further spares class by class while they fit.
+void layout_slots(lc_store* st) {
+    const size_t nc = st->class_bytes.size();
+    std::vector<size_t> order(nc);
+    for (size_t c = 0; c < nc; ++c) order[c] = c;
+    std::sort(order.begin(), order.end(),
+              [&](size_t a, size_t b) { return st->class_bytes[a] > st->class_bytes[b]; });
+    st->class_slots.assign(nc, 0);
+    st->class_free.assign(nc, {});
+    uint64_t top = 0;
+    auto place = [&](size_t c) -> bool {
+        const uint64_t z = st->class_bytes[c];
+        const uint64_t at = log_place(st, top, z);
+        if (at + z > st->capacity) return false;
+        st->class_free[c].push_back(at);
+        st->class_slots[c] += 1;
+        top = at + z;
+        return true;
+    };
+    for (size_t c : order)
+        for (int32_t k = 0; k <= st->class_layers[c]; ++k)
+            if (!place(c)) return;
+    for (bool grew = true; grew;) {
+        grew = false;
+        for (size_t c : order) grew = place(c) || grew;
+    }
+}
+
+// Newest-only mode: once a layer has a durable version, its older durable
+// versions are released (pending ones stay until they are durable).
+void store_release_superseded(lc_store* st) {
+    std::vector<int64_t> newest(size_t(st->nlayers), -1);
+    for (size_t i = 0; i < st->versions.size(); ++i) {
+        const StoreVersion& v = st->versions[i];
+        if (!v.durable) continue;
+        const int64_t cur = newest[size_t(v.layer)];
+        if (cur < 0 || v.step > st->versions[size_t(cur)].step ||
+            (v.step == st->versions[size_t(cur)].step && v.id > st->versions[size_t(cur)].id))
+            newest[size_t(v.layer)] = int64_t(i);
+    }
+    std::vector<StoreVersion> keep;
+    keep.reserve(st->versions.size());
+    for (size_t i = 0; i < st->versions.size(); ++i) {
+        const StoreVersion& v = st->versions[i];
+        if (v.durable && newest[size_t(v.layer)] != int64_t(i))
+            st->class_free[size_t(st->layer_class[size_t(v.layer)])].push_back(v.off);
+        else
+            keep.push_back(v);
+    }
+    st->versions.swap(keep);
+}
+
+}  // namespace
 
 struct PendingPack {
     int64_t step;
@@ -193,6 +276,7 @@ struct lc_ctx {
     bool bulk_sources = false;             // every registered array is device memory
     uint32_t* h_fault = nullptr;           // pinned, mapped: a bulk copy gave up waiting
     uint32_t* d_fault = nullptr;           // its device address
+    uint32_t* d_fault_dev = nullptr;       // its copy in device memory (read by every copy CTA)
     bool any_write_ref = false;
     std::vector<int32_t> order;            // measure position -> registration index
     bool snap_missing = false;             // some segment has no snapshot
@@ -241,6 +325,19 @@ struct lc_ctx {
     cudaStream_t capture_stream = nullptr;
     cudaGraphExec_t graph_exec = nullptr;
     lc_counters graph_delta{};             // what one replay of the graph launches
+
+    // copy trace: two timing events per staged chunk (lc_copy_trace_*)
+    struct Span {
+        int32_t kind;
+        int32_t chunk;
+        int64_t step;
+        uint64_t bytes;
+        cudaEvent_t a, b;
+    };
+    bool trace_on = false;
+    std::vector<Span> trace;
+    std::vector<cudaEvent_t> trace_pool;   // events of cleared records, for reuse
+    int64_t trace_dropped = 0;
 };
 
 namespace {
@@ -272,6 +369,7 @@ bool use_bulk(const lc_ctx* ctx, const void* base) {
 
 cudaError_t launch_copy_engine(lc_ctx* ctx, CopyParams p, bool bulk, uint64_t units, cudaStream_t s) {
     p.fault = ctx->d_fault;
+    p.fault_dev = ctx->d_fault_dev;
     p.stall_first = (ctx->cfg.debug_flags & LC_DEBUG_BULK_STALL) ? 1 : 0;
     const uint64_t cap = uint64_t(bulk ? ctx->bulk_grid : ctx->copy_grid);
     const int grid = int(std::max<uint64_t>(1, std::min<uint64_t>(cap, units)));
@@ -279,6 +377,50 @@ cudaError_t launch_copy_engine(lc_ctx* ctx, CopyParams p, bool bulk, uint64_t un
     ctx->counters.copy_launches += 1;
     if (bulk) ctx->counters.bulk_copy_launches += 1;
     return bulk ? launch_copy_bulk(p, grid, s) : launch_copy(p, grid, s);
+}
+
+// Copy trace.  A span's start event is recorded on its stream right before
+// the span's work and its end event right after, so end - start is the work
+// itself and a gap between spans of one stream is time that stream waited.
+// Tracing never makes a call fail: a span that cannot be recorded is dropped.
+constexpr size_t kMaxTraceSpans = size_t(1) << 16;
+
+cudaEvent_t trace_event(lc_ctx* ctx) {
+    if (!ctx->trace_pool.empty()) {
+        cudaEvent_t e = ctx->trace_pool.back();
+        ctx->trace_pool.pop_back();
+        return e;
+    }
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    return e;
+}
+
+int64_t trace_begin(lc_ctx* ctx, int32_t kind, int32_t chunk, int64_t step, uint64_t bytes, cudaStream_t s) {
+    if (!ctx->trace_on) return -1;
+    if (ctx->trace.size() >= kMaxTraceSpans) {
+        ctx->trace_dropped += 1;
+        return -1;
+    }
+    cudaEvent_t a = trace_event(ctx), b = a ? trace_event(ctx) : nullptr;
+    if (!a || !b || cudaEventRecord(a, s) != cudaSuccess) {
+        cudaGetLastError();
+        if (a) ctx->trace_pool.push_back(a);
+        if (b) ctx->trace_pool.push_back(b);
+        ctx->trace_dropped += 1;
+        return -1;
+    }
+    ctx->trace.push_back({kind, chunk, step, bytes, a, b});
+    return int64_t(ctx->trace.size()) - 1;
+}
+
+void trace_end(lc_ctx* ctx, int64_t idx, cudaStream_t s) {
+    if (idx < 0) return;
+    // a failed record leaves the span untimed (lc_copy_trace_read reports NaN)
+    if (cudaEventRecord(ctx->trace[size_t(idx)].b, s) != cudaSuccess) cudaGetLastError();
 }
 
 // The Eq. 1 scan on the context's engine.
@@ -363,6 +505,8 @@ extern "C" lc_status lc_create(lc_ctx** out, int device, void* cuda_stream, cons
         *ctx->h_fault = 0;
         e = cudaHostGetDevicePointer(reinterpret_cast<void**>(&ctx->d_fault), ctx->h_fault, 0);
     }
+    if (e == cudaSuccess) e = cudaMalloc(reinterpret_cast<void**>(&ctx->d_fault_dev), 16);
+    if (e == cudaSuccess) e = cudaMemset(ctx->d_fault_dev, 0, 16);
     int bocc = 0;
     if (e == cudaSuccess) e = copy_bulk_prepare(&bocc);
     if (e != cudaSuccess) {
@@ -392,9 +536,15 @@ extern "C" void lc_destroy(lc_ctx* ctx) {
         if (sl.host) cudaFreeHost(sl.host);
         if (sl.done) cudaEventDestroy(sl.done);
     }
+    for (auto& sp : ctx->trace) {
+        cudaEventDestroy(sp.a);
+        cudaEventDestroy(sp.b);
+    }
+    for (cudaEvent_t e : ctx->trace_pool) cudaEventDestroy(e);
     if (ctx->graph_exec) cudaGraphExecDestroy(ctx->graph_exec);
     if (ctx->capture_stream) cudaStreamDestroy(ctx->capture_stream);
     cudaFree(ctx->d_tables);
+    cudaFree(ctx->d_fault_dev);
     cudaFree(ctx->d_opt);
     cudaFree(ctx->d_staging);
     if (ctx->h_result) cudaFreeHost(ctx->h_result);
@@ -1052,20 +1202,75 @@ extern "C" lc_status lc_pack_async(lc_ctx* ctx, lc_store* st) {
     // the staging ring first: a failure leaves the store untouched
     LC_TRY(ensure_staging(ctx));
     // reserve the destination of every selected layer block in the store
-    struct Extent { uint64_t soff; uint8_t* host; uint64_t len; };
+    struct Extent { uint64_t soff; uint8_t* host; uint64_t len; int32_t layer; };
     std::vector<Extent> ext;
     std::vector<StoreVersion> fresh;
+    std::vector<std::vector<int32_t>> wait_before;   // newest-only: layers to see complete first
     if (st->per_layer == 0) {
-        if (st->top + bytes > st->capacity)
-            return fail(LC_ERR_CAPACITY, "lc_pack_async: store holds %llu of %llu bytes, %llu more needed",
-                        (unsigned long long)st->top, (unsigned long long)st->capacity,
-                        (unsigned long long)bytes);
-        ext.push_back({0, st->arena + st->top, bytes});
+        // each layer block goes to the next offset that touches no excluded
+        // range; blocks that land back to back share one extent
+        uint64_t cur = st->top;
         for (int32_t l = 0; l < ctx->nlayers; ++l) {
             if (!ctx->mask[l]) continue;
-            fresh.push_back({st->next_id++, l, 0, ctx->hdr.step, st->top + ctx->offsets[l], ctx->layer_bytes[l], -1});
+            const uint64_t lb = ctx->layer_bytes[l];
+            const uint64_t at = log_place(st, cur, lb);
+            if (at + lb > st->capacity)
+                return fail(LC_ERR_CAPACITY, "lc_pack_async: store holds %llu of %llu bytes, %llu more needed",
+                            (unsigned long long)st->top, (unsigned long long)st->capacity,
+                            (unsigned long long)bytes);
+            uint8_t* host = st->arena + at;
+            if (!ext.empty() && ext.back().soff + ext.back().len == ctx->offsets[l] &&
+                ext.back().host + ext.back().len == host)
+                ext.back().len += lb;
+            else
+                ext.push_back({ctx->offsets[l], host, lb, l});
+            fresh.push_back({0, l, 0, ctx->hdr.step, at, lb, -1});
+            cur = at + lb;
         }
-        st->top += bytes;
+        for (StoreVersion& v : fresh) v.id = st->next_id++;
+        st->top = cur;
+    } else if (st->per_layer == 1) {
+        // Newest-only: the placement of the step's blocks is decided here,
+        // before anything is enqueued.  Layers ascending take a free slot of
+        // their size class.  When the class has none, the earliest layer of
+        // the step in that class not yet counted complete is to be waited
+        // for: once its copy has landed its previous version's slot is free.
+        // With a spare slot per class every step fits; a CAPACITY error
+        // (fewer slots, after exclusions) leaves everything untouched.
+        for (const StoreVersion& v : st->versions)
+            if (!v.durable)
+                return fail(LC_ERR_STATE, "lc_pack_async: the newest-only store still holds a pending version "
+                                          "of layer %d (call lc_wait_durable)", v.layer);
+        std::vector<std::vector<uint64_t>> free = st->class_free;
+        std::vector<int64_t> old(size_t(ctx->nlayers), -1);
+        for (size_t i = 0; i < st->versions.size(); ++i) old[size_t(st->versions[i].layer)] = int64_t(i);
+        const size_t nc = st->class_bytes.size();
+        std::vector<std::vector<int32_t>> issued(nc);
+        std::vector<size_t> next_done(nc, 0);
+        wait_before.assign(size_t(ctx->nlayers), {});
+        for (int32_t l = 0; l < ctx->nlayers; ++l) {
+            if (!ctx->mask[l]) continue;
+            const size_t c = size_t(st->layer_class[size_t(l)]);
+            while (free[c].empty()) {
+                if (next_done[c] == issued[c].size())
+                    return fail(LC_ERR_CAPACITY,
+                                "lc_pack_async: no slot for the %llu-byte block of layer %d in the newest-only "
+                                "store (%d slots of that size for %d layers)",
+                                (unsigned long long)ctx->layer_bytes[l], l, st->class_slots[c],
+                                st->class_layers[c]);
+                const int32_t x = issued[c][next_done[c]++];
+                wait_before[size_t(l)].push_back(x);
+                if (old[size_t(x)] >= 0) free[c].push_back(st->versions[size_t(old[size_t(x)])].off);
+            }
+            const uint64_t off = free[c].back();
+            free[c].pop_back();
+            issued[c].push_back(l);
+            ext.push_back({ctx->offsets[l], st->arena + off, ctx->layer_bytes[l], l});
+            fresh.push_back({st->next_id++, l, 0, ctx->hdr.step, off, ctx->layer_bytes[l], -1});
+        }
+        // the free slots once every waited-for layer's old version is gone;
+        // the other old versions free theirs in lc_wait_durable
+        st->class_free.swap(free);
     } else {
         for (int32_t l = 0; l < ctx->nlayers; ++l) {
             if (!ctx->mask[l]) continue;
@@ -1082,7 +1287,7 @@ extern "C" lc_status lc_pack_async(lc_ctx* ctx, lc_store* st) {
                                               [&](const StoreVersion& v) { return v.layer == l && v.slot == slot; }),
                                st->versions.end());
             st->layer_writes[l] += 1;
-            ext.push_back({ctx->offsets[l], st->arena + off, ctx->layer_bytes[l]});
+            ext.push_back({ctx->offsets[l], st->arena + off, ctx->layer_bytes[l], l});
             fresh.push_back({st->next_id++, l, 0, ctx->hdr.step, off, ctx->layer_bytes[l], slot});
         }
     }
@@ -1094,6 +1299,28 @@ extern "C" lc_status lc_pack_async(lc_ctx* ctx, lc_store* st) {
                                           return true;
                                       }),
                        st->inflight.end());
+    // newest-only: an event after the copy that completes each layer's block,
+    // waited for (and the layer's version then counted durable) before a
+    // block that reuses the room of that layer's previous version is written
+    const bool newest = st->per_layer == 1;
+    std::vector<cudaEvent_t> layer_done(newest ? size_t(ctx->nlayers) : 0, nullptr);
+    std::vector<size_t> fresh_of(newest ? size_t(ctx->nlayers) : 0, 0);
+    for (size_t i = 0; i < fresh.size() && newest; ++i) fresh_of[size_t(fresh[i].layer)] = i;
+    auto drop_layer_events = [&]() {
+        for (cudaEvent_t e : layer_done)
+            if (e) cudaEventDestroy(e);
+    };
+    // a layer's copy has landed: its new version is durable, the old one is
+    // gone (its room was already counted free by the placement)
+    auto complete_layer = [&](int32_t x) -> lc_status {
+        lc_status rc = wait_event(layer_done[size_t(x)], ctx->cfg.timeout_ms, "lc_pack_async");
+        if (rc != LC_OK) return rc;
+        fresh[fresh_of[size_t(x)]].durable = 1;
+        st->versions.erase(std::remove_if(st->versions.begin(), st->versions.end(),
+                                          [&](const StoreVersion& v) { return v.layer == x; }),
+                           st->versions.end());
+        return LC_OK;
+    };
     // ring: gather chunk c into slot c%2 on the stream, copy it out on the copy stream
     const uint64_t S = ctx->slot_bytes;
     for (uint64_t lo = 0, c = 0; lo < bytes; lo += S, ++c) {
@@ -1101,19 +1328,46 @@ extern "C" lc_status lc_pack_async(lc_ctx* ctx, lc_store* st) {
         const uint64_t hi = std::min(bytes, lo + S);
         uint8_t* slot = ctx->d_staging + uint64_t(r) * S;
         if (ctx->slot_busy[r]) LC_CUDA(cudaStreamWaitEvent(ctx->stream, ctx->ev_slot_free[r], 0));
+        const int64_t tg = trace_begin(ctx, LC_SPAN_GATHER, int32_t(c), ctx->hdr.step, hi - lo, ctx->stream);
         LC_TRY(launch_copy_range(ctx, ctx->d_pack_desc, ctx->hdr.n_pack_desc, kGather, lo, hi, slot, ctx->stream));
+        trace_end(ctx, tg, ctx->stream);
         LC_CUDA(cudaEventRecord(ctx->ev_slot_filled[r], ctx->stream));
         LC_CUDA(cudaStreamWaitEvent(ctx->copy_stream, ctx->ev_slot_filled[r], 0));
+        const int64_t tc = trace_begin(ctx, LC_SPAN_D2H, int32_t(c), ctx->hdr.step, hi - lo, ctx->copy_stream);
         for (const Extent& e : ext) {
             const uint64_t a = std::max(lo, e.soff), b = std::min(hi, e.soff + e.len);
             if (a >= b) continue;
+            if (newest && a == e.soff) {
+                for (int32_t x : wait_before[size_t(e.layer)]) {
+                    const lc_status rc = complete_layer(x);
+                    if (rc != LC_OK) {
+                        // keep the versions whose copies are known complete; the
+                        // room of the others stays taken
+                        for (const StoreVersion& v : fresh)
+                            if (v.durable) st->versions.push_back(v);
+                        drop_layer_events();
+                        return rc;
+                    }
+                }
+            }
             LC_CUDA(cudaMemcpyAsync(e.host + (a - e.soff), slot + (a - lo), b - a, cudaMemcpyDeviceToHost,
                                     ctx->copy_stream));
             ctx->counters.d2h_bytes += b - a;
+            if (newest && b == e.soff + e.len) {
+                cudaError_t ee = cudaEventCreateWithFlags(&layer_done[size_t(e.layer)], cudaEventDisableTiming);
+                if (ee == cudaSuccess) ee = cudaEventRecord(layer_done[size_t(e.layer)], ctx->copy_stream);
+                if (ee != cudaSuccess) {
+                    cudaGetLastError();
+                    drop_layer_events();
+                    return fail(LC_ERR_CUDA, "lc_pack_async: %s", cudaGetErrorString(ee));
+                }
+            }
         }
+        trace_end(ctx, tc, ctx->copy_stream);
         LC_CUDA(cudaEventRecord(ctx->ev_slot_free[r], ctx->copy_stream));
         ctx->slot_busy[r] = true;
     }
+    drop_layer_events();
     PendingPack pp;
     pp.step = ctx->hdr.step;
     pp.store = st;
@@ -1169,6 +1423,7 @@ extern "C" lc_status lc_wait_durable(lc_ctx* ctx, int64_t step, int32_t timeout_
             if (g_live_stores.count(pp.store)) {
                 for (StoreVersion& v : pp.store->versions)
                     if (std::find(pp.ids.begin(), pp.ids.end(), v.id) != pp.ids.end()) v.durable = 1;
+                if (pp.store->per_layer == 1) store_release_superseded(pp.store);
             }
         }
         cudaEventDestroy(pp.done);
@@ -1439,6 +1694,7 @@ extern "C" lc_status lc_restore(lc_ctx* ctx, lc_store* st, int64_t t_fail, int64
         uint8_t* slot = ctx->d_staging + uint64_t(r) * S;
         cudaError_t e = cudaSuccess;
         if (ctx->slot_busy[r]) e = cudaStreamWaitEvent(ctx->copy_stream, ctx->ev_slot_free[r], 0);
+        const int64_t th = trace_begin(ctx, LC_SPAN_H2D, int32_t(c), t_fail, hi - lo, ctx->copy_stream);
         for (int32_t l = 0; l < N && e == cudaSuccess; ++l) {
             const uint64_t a = std::max(lo, soff[l]), b = std::min(hi, soff[l] + ctx->layer_bytes[l]);
             if (a >= b) continue;
@@ -1447,6 +1703,7 @@ extern "C" lc_status lc_restore(lc_ctx* ctx, lc_store* st, int64_t t_fail, int64
                                 cudaMemcpyHostToDevice, ctx->copy_stream);
             ctx->counters.h2d_bytes += b - a;
         }
+        trace_end(ctx, th, ctx->copy_stream);
         if (e == cudaSuccess) e = cudaEventRecord(ctx->ev_slot_filled[r], ctx->copy_stream);
         if (e == cudaSuccess) e = cudaStreamWaitEvent(ctx->stream, ctx->ev_slot_filled[r], 0);
         if (e != cudaSuccess) {
@@ -1454,7 +1711,9 @@ extern "C" lc_status lc_restore(lc_ctx* ctx, lc_store* st, int64_t t_fail, int64
             rc = fail(LC_ERR_CUDA, "lc_restore: %s", cudaGetErrorString(e));
             break;
         }
+        const int64_t ts = trace_begin(ctx, LC_SPAN_SCATTER, int32_t(c), t_fail, hi - lo, ctx->stream);
         rc = launch_copy_range(ctx, ctx->d_restore_desc, nsec, kScatter, lo, hi, slot, ctx->stream);
+        trace_end(ctx, ts, ctx->stream);
         if (rc == LC_OK && cudaEventRecord(ctx->ev_slot_free[r], ctx->stream) != cudaSuccess) {
             cudaGetLastError();
             rc = fail(LC_ERR_CUDA, "lc_restore: event record failed");
@@ -1506,6 +1765,53 @@ extern "C" lc_status lc_get_counters(const lc_ctx* ctx, lc_counters* out) {
 }
 
 // ---------------------------------------------------------------------------
+// copy trace
+// ---------------------------------------------------------------------------
+extern "C" lc_status lc_copy_trace_enable(lc_ctx* ctx, int32_t enable) {
+    g_err.clear();
+    if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_copy_trace_enable: ctx is NULL");
+    for (auto& sp : ctx->trace) {
+        ctx->trace_pool.push_back(sp.a);
+        ctx->trace_pool.push_back(sp.b);
+    }
+    ctx->trace.clear();
+    ctx->trace_dropped = 0;
+    ctx->trace_on = enable != 0;
+    return LC_OK;
+}
+
+extern "C" lc_status lc_copy_trace_read(lc_ctx* ctx, lc_copy_span* out, int64_t cap, int64_t* n_out,
+                                        int64_t* dropped_out) {
+    g_err.clear();
+    if (!ctx) return fail(LC_ERR_INVALID_ARG, "lc_copy_trace_read: ctx is NULL");
+    if (cap < 0 || (cap > 0 && !out)) return fail(LC_ERR_INVALID_ARG, "lc_copy_trace_read: bad output array");
+    if (n_out) *n_out = int64_t(ctx->trace.size());
+    if (dropped_out) *dropped_out = ctx->trace_dropped;
+    const size_t n = std::min(ctx->trace.size(), size_t(cap));
+    if (n == 0) return LC_OK;
+    DeviceGuard g(ctx->device);
+    for (size_t i = 0; i < n; ++i) {
+        LC_TRY(wait_event(ctx->trace[i].a, ctx->cfg.timeout_ms, "lc_copy_trace_read"));
+        LC_TRY(wait_event(ctx->trace[i].b, ctx->cfg.timeout_ms, "lc_copy_trace_read"));
+    }
+    const cudaEvent_t base = ctx->trace[0].a;
+    for (size_t i = 0; i < n; ++i) {
+        const lc_ctx::Span& sp = ctx->trace[i];
+        float a = 0.f, b = 0.f;
+        const bool ok = cudaEventElapsedTime(&a, base, sp.a) == cudaSuccess &&
+                        cudaEventElapsedTime(&b, base, sp.b) == cudaSuccess;
+        if (!ok) cudaGetLastError();
+        out[i].kind = sp.kind;
+        out[i].chunk = sp.chunk;
+        out[i].step = sp.step;
+        out[i].bytes = sp.bytes;
+        out[i].start_ms = ok ? double(a) : std::nan("");
+        out[i].end_ms = ok ? double(b) : std::nan("");
+    }
+    return LC_OK;
+}
+
+// ---------------------------------------------------------------------------
 // stores
 // ---------------------------------------------------------------------------
 extern "C" lc_status lc_store_create(lc_store** out, const lc_ctx* ctx, uint64_t capacity_bytes,
@@ -1514,8 +1820,8 @@ extern "C" lc_status lc_store_create(lc_store** out, const lc_ctx* ctx, uint64_t
     if (!out || !ctx) return fail(LC_ERR_INVALID_ARG, "lc_store_create: NULL argument");
     *out = nullptr;
     if (ctx->state == kNew) return fail(LC_ERR_STATE, "lc_store_create: no layout registered");
-    if (versions_per_layer < 0 || versions_per_layer == 1)
-        return fail(LC_ERR_INVALID_ARG, "lc_store_create: versions_per_layer must be 0 or >= 2");
+    if (versions_per_layer < 0)
+        return fail(LC_ERR_INVALID_ARG, "lc_store_create: versions_per_layer must be >= 0");
     lc_store* st = new lc_store();
     st->nlayers = ctx->nlayers;
     st->per_layer = versions_per_layer;
@@ -1526,6 +1832,32 @@ extern "C" lc_status lc_store_create(lc_store** out, const lc_ctx* ctx, uint64_t
             return fail(LC_ERR_INVALID_ARG, "lc_store_create: capacity_bytes must be > 0");
         }
         st->capacity = capacity_bytes;
+    } else if (versions_per_layer == 1) {
+        // size classes of the layer blocks; every layer's slot plus a spare per class
+        st->layer_class.assign(size_t(ctx->nlayers), -1);
+        uint64_t need = 0;
+        for (int32_t l = 0; l < ctx->nlayers; ++l) {
+            const uint64_t z = round_up(ctx->layer_bytes[size_t(l)], kStoreGrain);
+            size_t c = 0;
+            while (c < st->class_bytes.size() && st->class_bytes[c] != z) ++c;
+            if (c == st->class_bytes.size()) {
+                st->class_bytes.push_back(z);
+                st->class_layers.push_back(0);
+                need += z;
+            }
+            st->class_layers[c] += 1;
+            st->layer_class[size_t(l)] = int32_t(c);
+            need += z;
+        }
+        if (capacity_bytes < need) {
+            delete st;
+            return fail(LC_ERR_INVALID_ARG,
+                        "lc_store_create: a newest-only store needs capacity_bytes >= %llu (every layer's "
+                        "block plus one block of each distinct size), got %llu",
+                        (unsigned long long)need, (unsigned long long)capacity_bytes);
+        }
+        st->capacity = capacity_bytes / kStoreGrain * kStoreGrain;
+        layout_slots(st);
     } else {
         st->layer_base.resize(ctx->nlayers);
         st->layer_writes.assign(ctx->nlayers, 0);
@@ -1588,11 +1920,24 @@ extern "C" lc_status lc_store_clear(lc_store* st) {
     st->versions.clear();
     st->top = 0;
     std::fill(st->layer_writes.begin(), st->layer_writes.end(), 0);
+    if (st->per_layer == 1) layout_slots(st);
     return LC_OK;
 }
 
 extern "C" int64_t lc_store_num_versions(const lc_store* st) {
     return st ? int64_t(st->versions.size()) : 0;
+}
+
+extern "C" lc_status lc_store_get_info(const lc_store* st, lc_store_info* out) {
+    g_err.clear();
+    if (!st || !out) return fail(LC_ERR_INVALID_ARG, "lc_store_get_info: NULL argument");
+    std::memset(out, 0, sizeof *out);
+    out->arena = st->arena;
+    out->capacity = st->capacity;
+    for (const auto& x : st->excluded) out->excluded_bytes += x.second;
+    for (const StoreVersion& v : st->versions) out->used_bytes += v.bytes;
+    out->versions_per_layer = st->per_layer;
+    return LC_OK;
 }
 
 extern "C" lc_status lc_store_get_version(const lc_store* st, int64_t index, lc_version* out) {
@@ -1626,6 +1971,138 @@ extern "C" lc_status lc_store_plan(const lc_store* st, int64_t t_fail, int64_t* 
     return LC_OK;
 }
 
+extern "C" lc_status lc_store_exclude(lc_store* st, uint64_t offset, uint64_t bytes) {
+    g_err.clear();
+    if (!st) return fail(LC_ERR_INVALID_ARG, "lc_store_exclude: store is NULL");
+    if (st->per_layer >= 2)
+        return fail(LC_ERR_INVALID_ARG, "lc_store_exclude: a ring store's slots are fixed; use a log or "
+                                        "newest-only store");
+    if (bytes == 0 || offset >= st->capacity || bytes > st->capacity - offset)
+        return fail(LC_ERR_INVALID_ARG, "lc_store_exclude: range [%llu, +%llu) outside the %llu-byte arena",
+                    (unsigned long long)offset, (unsigned long long)bytes, (unsigned long long)st->capacity);
+    // whole 4096-byte granules, so newest-only blocks stay aligned
+    const uint64_t a = offset / kStoreGrain * kStoreGrain;
+    const uint64_t b = std::min(st->capacity, round_up(offset + bytes, kStoreGrain));
+    for (const StoreVersion& v : st->versions)
+        if (v.off < b && a < v.off + v.bytes)
+            return fail(LC_ERR_STATE, "lc_store_exclude: version of layer %d (step %lld) lies in the range",
+                        v.layer, (long long)v.step);
+    // merge into the excluded ranges
+    uint64_t lo = a, hi = b;
+    for (auto it = st->excluded.begin(); it != st->excluded.end();) {
+        if (it->first <= hi && lo <= it->first + it->second) {
+            lo = std::min(lo, it->first);
+            hi = std::max(hi, it->first + it->second);
+            it = st->excluded.erase(it);
+        } else {
+            ++it;
+        }
+    }
+    st->excluded.emplace(lo, hi - lo);
+    if (st->per_layer == 1) {
+        if (st->versions.empty()) {
+            layout_slots(st);          // an empty store lays its slots out anew
+        } else {
+            for (size_t c = 0; c < st->class_free.size(); ++c) {
+                auto& fl = st->class_free[c];
+                const uint64_t z = st->class_bytes[c];
+                const size_t before = fl.size();
+                fl.erase(std::remove_if(fl.begin(), fl.end(), [&](uint64_t o) { return o < hi && lo < o + z; }),
+                         fl.end());
+                st->class_slots[c] -= int32_t(before - fl.size());
+            }
+        }
+    }
+    return LC_OK;
+}
+
+extern "C" lc_status lc_store_check_dma(lc_store* st, lc_ctx* ctx, uint64_t region_bytes, int32_t passes,
+                                        double min_fraction, double* rates_out, int64_t rates_cap,
+                                        uint64_t* excluded_out) {
+    Range range("lc_store_check_dma");
+    g_err.clear();
+    if (!st || !ctx) return fail(LC_ERR_INVALID_ARG, "lc_store_check_dma: NULL argument");
+    if (st->per_layer >= 2) return fail(LC_ERR_INVALID_ARG, "lc_store_check_dma: ring stores are not supported");
+    if (region_bytes == 0) region_bytes = 256ull << 20;
+    if (region_bytes % kStoreGrain || region_bytes < (1ull << 20) || region_bytes > (1ull << 30))
+        return fail(LC_ERR_INVALID_ARG, "lc_store_check_dma: region_bytes must be a multiple of 4096 in [1 MiB, 1 GiB]");
+    if (!(min_fraction >= 0.0) || !std::isfinite(min_fraction))
+        return fail(LC_ERR_INVALID_ARG, "lc_store_check_dma: min_fraction must be finite and >= 0");
+    if (passes == 0) passes = 4;
+    if (passes < 1 || passes > 64) return fail(LC_ERR_INVALID_ARG, "lc_store_check_dma: passes must be in [1, 64]");
+    if (!st->versions.empty() || !st->inflight.empty())
+        return fail(LC_ERR_STATE, "lc_store_check_dma: the store must be empty (it overwrites the arena)");
+    const int64_t n = int64_t((st->capacity + region_bytes - 1) / region_bytes);
+    if (rates_out && rates_cap < n)
+        return fail(LC_ERR_INVALID_ARG, "lc_store_check_dma: rates_out needs %lld entries", (long long)n);
+    DeviceGuard g(ctx->device);
+    void* src = nullptr;
+    cudaStream_t s = nullptr;
+    std::vector<cudaEvent_t> ev(size_t(n) + 1, nullptr);
+    std::vector<double> best(size_t(n), 0.0), worst(size_t(n), 0.0);
+    lc_status rc = LC_OK;
+    cudaError_t e = cudaMalloc(&src, region_bytes);
+    if (e == cudaSuccess) e = cudaMemset(src, 0, region_bytes);
+    if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking);
+    for (size_t i = 0; i < ev.size() && e == cudaSuccess; ++i) e = cudaEventCreate(&ev[i]);
+    // several passes: slow regions come and go (the same regions, slow in
+    // about half of the passes on the hosts measured), so a region is judged
+    // by its worst pass against the median of the regions' best passes
+    for (int pass = 0; pass < passes && e == cudaSuccess && rc == LC_OK; ++pass) {
+        e = cudaEventRecord(ev[0], s);
+        for (int64_t i = 0; i < n && e == cudaSuccess; ++i) {
+            const uint64_t off = uint64_t(i) * region_bytes;
+            const uint64_t len = std::min(region_bytes, st->capacity - off);
+            e = cudaMemcpyAsync(st->arena + off, src, len, cudaMemcpyDeviceToHost, s);
+            if (e == cudaSuccess) e = cudaEventRecord(ev[size_t(i) + 1], s);
+        }
+        if (e != cudaSuccess) break;
+        rc = wait_event(ev[size_t(n)], ctx->cfg.timeout_ms, "lc_store_check_dma");
+        for (int64_t i = 0; i < n && rc == LC_OK && e == cudaSuccess; ++i) {
+            float ms = 0.f;
+            e = cudaEventElapsedTime(&ms, ev[size_t(i)], ev[size_t(i) + 1]);
+            const uint64_t len = std::min(region_bytes, st->capacity - uint64_t(i) * region_bytes);
+            if (e == cudaSuccess && ms > 0.f) {
+                const double r = len / (1e6 * ms);
+                best[size_t(i)] = std::max(best[size_t(i)], r);
+                worst[size_t(i)] = pass == 0 ? r : std::min(worst[size_t(i)], r);
+            }
+        }
+    }
+    if (e != cudaSuccess && rc == LC_OK) {
+        cudaGetLastError();
+        rc = fail(LC_ERR_CUDA, "lc_store_check_dma: %s", cudaGetErrorString(e));
+    }
+    if (rc == LC_ERR_TIMEOUT) {
+        // copies still in flight: leave the source buffer to them rather than
+        // block in cudaFree (which waits for the whole device)
+        cudaGetLastError();
+        return rc;
+    }
+    if (s) cudaStreamSynchronize(s);
+    for (cudaEvent_t x : ev)
+        if (x) cudaEventDestroy(x);
+    if (s) cudaStreamDestroy(s);
+    if (src) cudaFree(src);
+    cudaGetLastError();
+    if (rc != LC_OK) return rc;
+    std::vector<double> sorted = best;
+    std::sort(sorted.begin(), sorted.end());
+    const double median = sorted[sorted.size() / 2];
+    uint64_t excluded = 0;
+    for (int64_t i = 0; i < n; ++i) {
+        if (rates_out) rates_out[i] = worst[size_t(i)];
+        if (worst[size_t(i)] < min_fraction * median) {
+            const uint64_t off = uint64_t(i) * region_bytes;
+            const uint64_t len = std::min(region_bytes, st->capacity - off);
+            LC_TRY(lc_store_exclude(st, off, len));
+            excluded += len;
+        }
+    }
+    if (excluded_out) *excluded_out = excluded;
+    return LC_OK;
+}
+
 // ---------------------------------------------------------------------------
 // host internals used by the file tier (lc_files.cu)
 // ---------------------------------------------------------------------------
@@ -1636,10 +2113,11 @@ const uint64_t* lc::store_layer_bytes(const lc_store* st) { return st->layer_byt
 uint8_t* lc::store_append(lc_store* st, int32_t layer, int64_t* index_out) {
     if (st->per_layer != 0 || layer < 0 || layer >= st->nlayers) return nullptr;
     const uint64_t bytes = st->layer_bytes[size_t(layer)];
-    if (st->top + bytes > st->capacity) return nullptr;
-    st->versions.push_back({st->next_id++, layer, 1, -1, st->top, bytes, -1});
-    uint8_t* p = st->arena + st->top;
-    st->top += bytes;
+    const uint64_t at = log_place(st, st->top, bytes);
+    if (at + bytes > st->capacity) return nullptr;
+    st->versions.push_back({st->next_id++, layer, 1, -1, at, bytes, -1});
+    uint8_t* p = st->arena + at;
+    st->top = at + bytes;
     if (index_out) *index_out = int64_t(st->versions.size()) - 1;
     return p;
 }

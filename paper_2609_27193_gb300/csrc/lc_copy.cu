@@ -339,6 +339,16 @@ struct BulkRing {
     BulkJob jobs[kStages];
 };
 
+// A bounded wait ran out: the host-mapped word tells the host, the device
+// copy tells the CTAs that start after this one.
+__device__ __forceinline__ void raise_copy_fault(const CopyParams& p) {
+    raise_fault(p.fault);
+    if (p.fault_dev) {
+        *reinterpret_cast<volatile uint32_t*>(p.fault_dev) = 1u;
+        __threadfence();
+    }
+}
+
 __device__ void bulk_produce(const CopyParams& p, int i, uint64_t x, uint64_t xe, uint32_t ring_s, BulkRing& r) {
     const uint32_t full_s = smem_addr(r.full), empty_s = smem_addr(r.empty);
     const uint64_t pol = evict_first_policy();
@@ -368,7 +378,7 @@ __device__ void bulk_produce(const CopyParams& p, int i, uint64_t x, uint64_t xe
         have = bulk_next_chunk(p, c, xe, j);
     }
     if (!ok) {
-        raise_fault(p.fault);
+        raise_copy_fault(p);
         // the loads of the last kStages chunks may still be landing in shared memory
         const uint64_t first = k > uint64_t(kStages) ? k - kStages : 0;
         for (uint64_t c = first; c < k; ++c)
@@ -382,7 +392,7 @@ __device__ void bulk_consume(const CopyParams& p, uint32_t ring_s, BulkRing& r) 
     for (uint64_t k = 0;; ++k) {
         const int s = int(k % kStages);
         if (!mbar_wait_bounded(full_s + 8 * s, uint32_t((k / kStages) & 1), kWaitNs)) {
-            raise_fault(p.fault);
+            raise_copy_fault(p);
             break;
         }
         const BulkJob j = r.jobs[s];
@@ -403,10 +413,14 @@ __device__ void bulk_consume(const CopyParams& p, uint32_t ring_s, BulkRing& r) 
 __global__ void __launch_bounds__(kCopyThreads, 1) copy_bulk_kernel(CopyParams p) {
     extern __shared__ __align__(128) uint8_t ring[];
     __shared__ __align__(8) BulkRing r;
+    __shared__ uint32_t s_abort;
     uint64_t x, xe;
     int first;
     if (!cta_range(p, x, xe, first)) return;
     if (threadIdx.x == 0) {
+        // an earlier CTA of this context gave up waiting: the copy's bytes
+        // are lost anyway, so this CTA does not start a wait of its own
+        s_abort = p.fault_dev ? *reinterpret_cast<volatile const uint32_t*>(p.fault_dev) : 0u;
         for (int s = 0; s < kStages; ++s) {
             mbar_init(smem_addr(&r.full[s]), 1);
             mbar_init(smem_addr(&r.empty[s]), 1);
@@ -414,6 +428,7 @@ __global__ void __launch_bounds__(kCopyThreads, 1) copy_bulk_kernel(CopyParams p
         mbar_init_fence();
     }
     __syncthreads();
+    if (s_abort) return;
     if (threadIdx.x < 64) {
         if (threadIdx.x == 0) bulk_produce(p, first, x, xe, smem_addr(ring), r);
         else if (threadIdx.x == 32) bulk_consume(p, smem_addr(ring), r);

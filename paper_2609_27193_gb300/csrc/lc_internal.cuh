@@ -91,6 +91,10 @@ struct CopyParams {
     // Host-mapped word a bulk-engine copy sets to 1 when a bounded wait
     // runs out (never cleared by the device).
     uint32_t* fault;
+    // Its copy in device memory, set together with it: every CTA of a bulk
+    // copy reads it before its first load and returns at once if it is set,
+    // so the later waves of a launch whose first wave gave up end at once.
+    uint32_t* fault_dev;
     // Test of that bound: each CTA's first bulk load announces 16 bytes more
     // than it brings, so its wait can only run out.
     int32_t stall_first;
