@@ -11,6 +11,8 @@
   store; at steps 50, 100 and 200 the run fails over: lc_restore writes
   the composite and the device state is compared with the oracle's
   composite bit for bit, then the run continues from it.
+* The same on the full 35-layer 8B layout with a bf16 matmul loop running
+  on another stream throughout, through a newest-only store.
 """
 import numpy as np
 import pytest
@@ -145,6 +147,135 @@ def test_cadence_regimes_with_failovers():
     assert regimes == set(wl.regimes)
     store.close()
     lc.close()
+
+
+def _bits(t):
+    """A tensor's raw bit pattern (so -0.0 and 0.0 differ)."""
+    torch = require_gpu()
+    return t.view(torch.int16) if t.element_size() == 2 else t.view(torch.int32)
+
+
+def test_cadence_full_8b_layout_under_gemm_load():
+    """The cadence workload at its full shape and load: the 35-layer
+    Llama-3-8B layout (1.05 GB embed and lm_head weights) for 200 steps with
+    the drift regimes switching every 50 steps, a bf16 8192^3 matmul loop on
+    another stream all along, and the library on a side stream persisting
+    through a newest-only pinned store.  On every step the selection rule is
+    re-checked on the CPU from the device's u (select-only).  At steps 50,
+    100 and 200 the run fails over: lc_restore writes the composite of §3.5 /
+    Eq. 8 (under the matmul load as well), and
+
+    * the chosen steps equal the oracle's pick over the durable versions;
+    * every tensor's W, R, exp_avg and exp_avg_sq equal, bit for bit, the
+      state captured when the oracle's picked version was persisted;
+    * for the embedding, a middle block and lm_head the store's block equals
+      the oracle's packed block of that state (§3.1) byte for byte, and the
+      restored tensors equal the oracle's unpacked composite;
+
+    then the run continues from the composite."""
+    torch = require_gpu()
+    import paper_2609_27193_gb300 as P
+    wl = WORKLOADS["8b-cadence"]
+    shape = wl.shape()
+    N = shape.nlayers
+    st = gen.SyntheticState(shape, device="cuda", seed=wl.seed)
+    K, tau = wl.max_staleness, wl.tau
+    main = torch.cuda.current_stream()
+    side = torch.cuda.Stream()
+    lc = make_lc(st, stream=side)
+    run = OracleRun(st.tensor_layer, st.numels, st.nlayers, st.dtypes, st.has_moments, keep_blocks="latest")
+    layer_tensors = run.layer_tensors
+    blocks = [lc.layer_block_bytes(l) for l in range(N)]
+    full = sum(blocks)
+    sizes = sorted({-(-b // 4096) * 4096 for b in blocks})
+    store = P.Store(lc, capacity_bytes=full + 2 * sum(sizes) + (1 << 30), versions_per_layer=1)
+    # the state of every layer as it was when last persisted
+    EW = [torch.empty_like(w) for w in st.W]
+    EM = [torch.empty_like(m) for m in st.m]
+    EV = [torch.empty_like(v) for v in st.v]
+    gs = torch.cuda.Stream()
+    a = torch.randn(8192, 8192, device="cuda", dtype=torch.bfloat16)
+    b = torch.randn(8192, 8192, device="cuda", dtype=torch.bfloat16)
+    c = torch.empty_like(a)
+
+    def gemm_burst(n=40):
+        with torch.cuda.stream(gs):
+            for _ in range(n):
+                torch.matmul(a, b, out=c)
+
+    def capture(mask):
+        for l in np.flatnonzero(mask):
+            for k in layer_tensors[l]:
+                EW[k].copy_(st.W[k])
+                EM[k].copy_(st.m[k])
+                EV[k].copy_(st.v[k])
+
+    def persist(mask, t):
+        capture(mask)
+        lc.pack_async(store)
+        lc.commit_snapshot()
+        lc.wait_durable(t)
+        run.record(mask, t)
+        run.mark_durable(t)
+        main.wait_stream(side)
+
+    sample = [0, N // 2, N - 1]
+    side.wait_stream(main)
+    gemm_burst()
+    lc.measure(0)
+    mask, u, _ = lc.select(tau, 0)
+    assert mask.all()
+    O.select_step(u, run.delta, run.t_last, tau, 0, 0)
+    persist(mask, 0)
+    regimes, persisted = set(), []
+    for t in range(1, 201):
+        scales, regime = cadence_scales(wl, shape, t)
+        regimes.add(regime)
+        st.drift(t, scales)
+        side.wait_stream(main)
+        gemm_burst()
+        lc.measure(t)
+        mask, u, nbytes = lc.select(tau, K)
+        omask, _, _ = O.select_step(u, run.delta, run.t_last, tau, K, t)
+        assert np.array_equal(mask, omask), "select-only check at step %d (%s)" % (t, regime)
+        persisted.append(nbytes)
+        persist(mask, t)
+        if t in (50, 100, 200):
+            gemm_burst()
+            steps = lc.restore(store, t)
+            pick = run.pick(t)
+            assert steps.tolist() == [run.versions[p]["step"] for p in pick], t
+            assert min(steps) >= t - K + 1
+            torch.cuda.synchronize()
+            for k in range(len(shape.tensors)):
+                for got, want, what in ((st.W[k], EW[k], "W"), (st.R[k], EW[k], "R"),
+                                        (st.m[k], EM[k], "exp_avg"), (st.v[k], EV[k], "exp_avg_sq")):
+                    assert torch.equal(_bits(got), _bits(want)), "%s of tensor %d at step %d" % (what, k, t)
+            spick = store.plan(t)
+            for l in sample:
+                ts = [O.Tensor(gen.SyntheticState.to_numpy(EW[k]), None, gen.SyntheticState.to_numpy(EM[k]),
+                               gen.SyntheticState.to_numpy(EV[k])) for k in layer_tensors[l]]
+                block = O.pack_layer(ts, run.align)
+                v = store.version(int(spick[l]))
+                assert v["step"] == steps[l] and v["bytes"] == block.size
+                assert np.array_equal(store.block(int(spick[l])), block), "block of layer %d at %d" % (l, t)
+                shp = run._shape_tensors(l)
+                O.unpack_layer(block, shp, run.align)
+                for k, ex in zip(layer_tensors[l], shp):
+                    assert np.array_equal(st.host("W", k), ex.w) and np.array_equal(st.host("R", k), ex.w)
+                    assert np.array_equal(st.host("m", k), ex.m) and np.array_equal(st.host("v", k), ex.v)
+                del ts, block, shp
+            # after a recovery each layer carries its version's step and no drift
+            run.t_last[:] = steps
+            run.delta[:] = 0.0
+            st.resync_master()
+    assert regimes == set(wl.regimes)
+    assert len(store) == N
+    assert sum(persisted) > 0
+    store.close()
+    lc.close()
+    del st, EW, EM, EV, a, b, c
+    torch.cuda.empty_cache()
 
 
 def test_llama8b_fused_adamw_sampled_parity():
