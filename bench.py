@@ -72,6 +72,9 @@ def parse_args():
                     help="write every span of the library's copy trace in the e2e loop and the "
                          "restore (per staging chunk: kind, step, bytes, start/end ms) to FILE "
                          "as JSON lines")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the short passes over the other workloads (tiny, 1b, 8b at tau 5e-4 "
+                         "and 2e-3, 8b-tensor, 8b-cadence) that the default 8b run adds as `configs`")
     ap.add_argument("--no-dma-check", action="store_true",
                     help="do not run lc_store_check_dma on the e2e store (by default the pinned "
                          "regions the GPU copies into at under half the median rate are kept out of use)")
@@ -469,6 +472,148 @@ def d2h_link_probe(torch, dev, nbytes=4 << 30):
     return best
 
 
+def config_pass(P, torch, dev, st, units, nunits, tau, K, steps, warmup, scales_for, dst, hbm,
+                per_tensor=False, gemm=None, regime_of=None, l2_bytes=128 << 20):
+    """One short device-resident pass over a workload: a fresh context whose
+    base state is the tensors as they are, then `warmup` untimed and `steps`
+    timed steps of drift -> measure -> select -> pack into device memory ->
+    fused commit (the headline step), CUDA events on the library's stream.
+    units[k] is the selection unit of tensor k; scales_for(i) the drift
+    scales of step i (per unit, or per tensor with per_tensor)."""
+    import numpy as np
+    side = torch.cuda.Stream(device=dev)
+    main = torch.cuda.current_stream(dev)
+    lc = P.LayerCheck(device=dev.index or 0, stream=side)
+    lc.register_layout([P.segment(units[k], st.W[k], st.R[k], st.m[k], st.v[k]) for k in range(len(units))],
+                       nunits)
+    payload, wbytes = [0] * nunits, [0] * nunits
+    mbytes = 0
+    for k, spec in enumerate(st.specs):
+        esz = 2 if st.dtypes[k] == "bf16" else 4
+        payload[units[k]] += spec.numel * esz + (8 * spec.numel if st.has_moments[k] else 0)
+        wbytes[units[k]] += spec.numel * esz
+        mbytes += 2 * spec.numel * esz
+    flush = torch.empty(4 * l2_bytes, dtype=torch.uint8, device=dev) if mbytes < 4 * l2_bytes else None
+    recs = []
+    for i in range(warmup + steps):
+        sc = scales_for(i)
+        if per_tensor:
+            st.drift(1000 + i, None, tensor_scale=sc)
+        else:
+            st.drift(1000 + i, sc)
+        if flush is not None:
+            flush.fill_(i & 0xFF)
+        side.wait_stream(main)
+        main.synchronize()
+        if gemm is not None:
+            gs, a, b, c = gemm
+            with torch.cuda.stream(gs):
+                for _ in range(40):
+                    torch.matmul(a, b, out=c)
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        h0 = time.perf_counter()
+        ev[0].record(side)
+        lc.measure(i + 1)
+        ev[1].record(side)
+        mask, u, nbytes = lc.select(tau, K)
+        h1 = time.perf_counter()
+        ev[2].record(side)
+        lc.pack_device(dst)
+        lc.commit_snapshot()
+        ev[3].record(side)
+        if i >= warmup:
+            recs.append((ev, h1 - h0, mask, nbytes, i))
+        main.wait_stream(side)
+    torch.cuda.synchronize()
+    lc.close()
+    l2_note = "L2 flushed before every step" if flush is not None else "inputs larger than L2"
+    del flush
+    el = lambda r, a, b: r[0][a].elapsed_time(r[0][b])
+    meas = [el(r, 0, 1) for r in recs]
+    pack = [el(r, 2, 3) for r in recs]
+    step = [el(r, 0, 3) for r in recs]
+    pbytes = [sum(2 * payload[l] + wbytes[l] for l in np.flatnonzero(r[2])) for r in recs]
+    dec = [1e3 * r[1] for r in recs]
+    mean = lambda x: sum(x) / len(x)
+    out = {"steps": steps, "warmup": warmup, "tau": tau, "max_staleness": K, "units": nunits,
+           "params": int(sum(s.numel for s in st.specs)),
+           "value": (mbytes * len(recs) + sum(pbytes)) / (sum(step) / 1e3) / 1e9, "unit": "GB/s",
+           "ms_per_step": mean(step), "decision_ms_p50": float(np.median(dec)),
+           "decision_ms_p99": float(np.percentile(dec, 99)),
+           "measure_ms": mean(meas), "measure_frac": mbytes / (mean(meas) / 1e3) / 1e9 / hbm,
+           "pack_ms": mean(pack),
+           "pack_frac": (mean(pbytes) / (mean(pack) / 1e3) / 1e9 / hbm) if mean(pack) > 0 else None,
+           "selected_fraction": float(np.mean([r[2].mean() for r in recs])),
+           "persisted_GB_per_step": mean([r[3] for r in recs]) / 1e9,
+           "l2": l2_note}
+    if regime_of is not None:
+        groups = {}
+        for r, ms_, pb in zip(recs, step, pbytes):
+            g = groups.setdefault(regime_of(r[4]), {"sel": [], "bytes": [], "ms": [], "dec": []})
+            g["sel"].append(float(r[2].mean()))
+            g["bytes"].append(r[3])
+            g["ms"].append(ms_)
+            g["dec"].append(1e3 * r[1])
+        out["regimes"] = {n: {"steps": len(g["ms"]), "selected_fraction": mean(g["sel"]),
+                              "persisted_GB_per_step": mean(g["bytes"]) / 1e9, "step_ms": mean(g["ms"]),
+                              "decision_ms_p50": float(np.median(g["dec"]))} for n, g in groups.items()}
+    return out
+
+
+def config_passes(P, torch, dev, st8, dst, hbm, l2_bytes):
+    """The other workloads beside the headline (8b at tau 1e-3): tiny, 1b,
+    8b at tau 5e-4 and 2e-3, the 291-unit per-tensor layout, and the
+    cadence workload's 200 steps with its matmul loop and drift regimes.
+    The 8B passes reuse the headline's tensors, each with a fresh context."""
+    from lc_workloads import gen
+    from lc_workloads.configs import WORKLOADS, cadence_scales
+    out = {}
+    w8 = WORKLOADS["8b"]
+    s8 = w8.shape()
+    sc8 = w8.layer_scales(s8)
+    units8 = [t.layer for t in s8.tensors]
+    for tau in (5e-4, 2e-3):
+        t0 = time.perf_counter()
+        out["8b tau=%g" % tau] = config_pass(P, torch, dev, st8, units8, s8.nlayers, tau, w8.max_staleness, 10, 3,
+                                             lambda i: sc8, dst, hbm, l2_bytes=l2_bytes)
+        out["8b tau=%g" % tau]["wall_s"] = time.perf_counter() - t0
+    wt = WORKLOADS["8b-tensor"]
+    st_shape = wt.shape()
+    sct = wt.layer_scales(st_shape)
+    t0 = time.perf_counter()
+    out["8b-tensor"] = config_pass(P, torch, dev, st8, list(range(len(st_shape.tensors))), st_shape.nlayers,
+                                   wt.tau, wt.max_staleness, 10, 3, lambda i: sct, dst, hbm, per_tensor=True,
+                                   l2_bytes=l2_bytes)
+    out["8b-tensor"]["wall_s"] = time.perf_counter() - t0
+    wc = WORKLOADS["8b-cadence"]
+    a = torch.randn(8192, 8192, device=dev, dtype=torch.bfloat16)
+    b = torch.randn(8192, 8192, device=dev, dtype=torch.bfloat16)
+    gemm = (torch.cuda.Stream(device=dev), a, b, torch.empty_like(a))
+    warm = 3
+    step_of = lambda i: max(1, i - warm + 1)       # timed steps 1..200
+    t0 = time.perf_counter()
+    out["8b-cadence"] = config_pass(P, torch, dev, st8, units8, s8.nlayers, wc.tau, wc.max_staleness, 200, warm,
+                                    lambda i: cadence_scales(wc, s8, step_of(i))[0], dst, hbm, gemm=gemm,
+                                    regime_of=lambda i: cadence_scales(wc, s8, step_of(i))[1],
+                                    l2_bytes=l2_bytes)
+    out["8b-cadence"]["wall_s"] = time.perf_counter() - t0
+    del a, b, gemm
+    for name in ("1b", "tiny"):
+        wl = WORKLOADS[name]
+        sh = wl.shape()
+        st = gen.SyntheticState(sh, device=dev, seed=wl.seed)
+        sc = wl.layer_scales(sh)
+        t0 = time.perf_counter()
+        out[name] = config_pass(P, torch, dev, st, [t.layer for t in sh.tensors], sh.nlayers, wl.tau,
+                                wl.max_staleness, 10, 3, lambda i: sc, dst, hbm, l2_bytes=l2_bytes)
+        out[name]["wall_s"] = time.perf_counter() - t0
+        del st
+        torch.cuda.empty_cache()
+    for name, d in out.items():
+        d["workload"] = name
+    return out
+
+
 def load_package():
     import paper_2609_27193_gb300 as P
     try:
@@ -849,6 +994,12 @@ def run_ours(args):
             e2e["files"] = ({"skipped": files_note} if files_note
                             else files_recovery(P, lc, args.files, t, f_bytes, f_s))
 
+    configs = None
+    if (world == 1 and not args.no_configs and args.workload == "8b" and args.path == "scan"
+            and args.drift == "snapshot" and not args.shape_blocks and args.tau is None
+            and args.copy_engine == "bulk"):
+        configs = config_passes(P, torch, dev, st, dst, hbm, l2_bytes)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         del dst
@@ -885,6 +1036,8 @@ def run_ours(args):
         "bulk_copy_launches": int(c1["bulk_copy_launches"] - c0["bulk_copy_launches"]),
         "capacity_overflow_steps": overflow,
         "regimes": regimes,
+        # short passes over the other workloads (device-resident, like value)
+        "configs": configs,
         "clocks": clk, "timed_wall_s_with_input_generation": wall, "setup_s": setup_s,
     }
     if rank == 0:
