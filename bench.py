@@ -911,12 +911,10 @@ def run_ours(args):
                              "excluded_bytes": int(excluded), "excluded_regions": int(excluded // region),
                              "worst_pass_GBps_median": float(srt[srt.size // 2]),
                              "worst_pass_GBps_p10": float(srt[srt.size // 10]), "worst_pass_GBps_min": float(srt[0]),
-                             "capacity": int(cap), "s": time.perf_counter() - tchk}
-                if cap - excluded < full:
-                    # too little room left for a full step: keep every region
-                    store.close()
-                    store = P.Store(lc, capacity_bytes=cap)
-                    dma_check["dropped"] = "exclusions would leave less than the full state; none applied"
+                             "capacity": int(cap), "s": time.perf_counter() - tchk,
+                             # slow regions whose exclusion would leave no room for a
+                             # step that persists every layer stay in use
+                             "rule": "slowest first, while a full step still fits"}
         link = d2h_link_probe(torch, dev)
         e_recs, e_bytes = [], []
         f_bytes, f_s = 0, 0.0

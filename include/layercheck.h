@@ -476,10 +476,16 @@ lc_status lc_store_exclude(lc_store* store, uint64_t offset, uint64_t bytes);
  * pinned arena copying at 15-60 GB/s in about half of the passes over it,
  * the rest at 193 GB/s in every pass).  This times `passes` device->host
  * copies into every region_bytes region of an empty log or newest-only
- * store (from a device buffer on ctx's device) and excludes
- * (lc_store_exclude) every region whose slowest pass ran below min_fraction
- * times the median of the regions' fastest passes.  region_bytes: 0 (256
- * MiB) or a multiple of 4096 in [1 MiB, 1 GiB]; passes: 0 (4) or 1..64.
+ * store (from a device buffer on ctx's device).  A region is slow if its
+ * slowest pass ran below min_fraction times the median of the regions'
+ * fastest passes.  The slow regions are excluded (lc_store_exclude) one at
+ * a time, slowest first (the lower index first on a tie), except that one
+ * whose exclusion would leave no room for a step that persists every layer
+ * stays in use: every layer's block in layer order from offset 0 (log
+ * store), or each block size's slots for its layers plus the spare
+ * (newest-only store).  A store that lacks that room before the call loses
+ * every slow region.  region_bytes: 0 (256 MiB) or a multiple of 4096 in
+ * [1 MiB, 1 GiB]; passes: 0 (4) or 1..64.
  * rates_out (host, nullable): each of the ceil(capacity / region_bytes)
  * regions' slowest GB/s; excluded_out (nullable): bytes excluded.
  * Overwrites the arena; blocks (bounded by ctx's timeout_ms).

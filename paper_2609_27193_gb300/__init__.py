@@ -392,8 +392,10 @@ class Store:
     def check_dma(self, lc, region_bytes=256 << 20, min_fraction=0.5, passes=4):
         """Time `passes` device->host copies into every region of the (empty)
         arena and exclude the regions whose slowest pass ran below
-        min_fraction x the median of the regions' fastest passes.  Returns
-        (each region's slowest GB/s as a numpy array, excluded bytes)."""
+        min_fraction x the median of the regions' fastest passes, slowest
+        first, as long as a step that persists every layer still fits.
+        Returns (each region's slowest GB/s as a numpy array, excluded
+        bytes)."""
         cap = int(self.capacity)
         n = -(-cap // int(region_bytes))
         rates = np.zeros(n, dtype=np.float64)

@@ -176,11 +176,12 @@ namespace {
 // Blocks of a newest-only store start on this boundary.
 constexpr uint64_t kStoreGrain = 4096;
 
-// Log mode: the first offset >= `from` at which `len` bytes touch no
-// excluded range.
-uint64_t log_place(const lc_store* st, uint64_t from, uint64_t len) {
+using RangeMap = std::map<uint64_t, uint64_t>;   // offset -> length, disjoint
+
+// The first offset >= `from` at which `len` bytes touch no range of `excl`.
+uint64_t place_around(const RangeMap& excl, uint64_t from, uint64_t len) {
     uint64_t at = from;
-    for (const auto& x : st->excluded) {
+    for (const auto& x : excl) {
         if (x.first + x.second <= at) continue;
         if (at + len <= x.first) break;
         at = x.first + x.second;
@@ -188,15 +189,66 @@ uint64_t log_place(const lc_store* st, uint64_t from, uint64_t len) {
     return at;
 }
 
-// Newest-only mode: lays the slots out in an empty store, skipping excluded
-// ranges -- classes largest first, each its layers' slots plus one spare,
-// then further spares class by class while they fit.
-void layout_slots(lc_store* st) {
+// Log mode: the first offset >= `from` at which `len` bytes touch no
+// excluded range.
+uint64_t log_place(const lc_store* st, uint64_t from, uint64_t len) {
+    return place_around(st->excluded, from, len);
+}
+
+// Adds [lo, hi) to `r`, merging it with the ranges it touches.
+void add_range(RangeMap& r, uint64_t lo, uint64_t hi) {
+    for (auto it = r.begin(); it != r.end();) {
+        if (it->first <= hi && lo <= it->first + it->second) {
+            lo = std::min(lo, it->first);
+            hi = std::max(hi, it->first + it->second);
+            it = r.erase(it);
+        } else {
+            ++it;
+        }
+    }
+    r.emplace(lo, hi - lo);
+}
+
+// Newest-only mode: size classes in the order their slots are laid out
+// (largest first; classes have distinct sizes).
+std::vector<size_t> classes_largest_first(const lc_store* st) {
     const size_t nc = st->class_bytes.size();
     std::vector<size_t> order(nc);
     for (size_t c = 0; c < nc; ++c) order[c] = c;
     std::sort(order.begin(), order.end(),
               [&](size_t a, size_t b) { return st->class_bytes[a] > st->class_bytes[b]; });
+    return order;
+}
+
+// Whether the store, empty and with `excl` out of use, takes a step that
+// persists every layer: in a log store every layer's block in layer order
+// from offset 0; in a newest-only store each size class's slots for its
+// layers plus its spare (the first pass of layout_slots).
+bool full_step_fits(const lc_store* st, const RangeMap& excl) {
+    uint64_t top = 0;
+    auto put = [&](uint64_t z) {
+        const uint64_t at = place_around(excl, top, z);
+        if (at + z > st->capacity) return false;
+        top = at + z;
+        return true;
+    };
+    if (st->per_layer == 0) {
+        for (uint64_t z : st->layer_bytes)
+            if (!put(z)) return false;
+        return true;
+    }
+    for (size_t c : classes_largest_first(st))
+        for (int32_t k = 0; k <= st->class_layers[c]; ++k)
+            if (!put(st->class_bytes[c])) return false;
+    return true;
+}
+
+// Newest-only mode: lays the slots out in an empty store, skipping excluded
+// ranges -- classes largest first, each its layers' slots plus one spare,
+// then further spares class by class while they fit.
+void layout_slots(lc_store* st) {
+    const size_t nc = st->class_bytes.size();
+    const std::vector<size_t> order = classes_largest_first(st);
     st->class_slots.assign(nc, 0);
     st->class_free.assign(nc, {});
     uint64_t top = 0;
@@ -1987,18 +2039,8 @@ extern "C" lc_status lc_store_exclude(lc_store* st, uint64_t offset, uint64_t by
         if (v.off < b && a < v.off + v.bytes)
             return fail(LC_ERR_STATE, "lc_store_exclude: version of layer %d (step %lld) lies in the range",
                         v.layer, (long long)v.step);
-    // merge into the excluded ranges
-    uint64_t lo = a, hi = b;
-    for (auto it = st->excluded.begin(); it != st->excluded.end();) {
-        if (it->first <= hi && lo <= it->first + it->second) {
-            lo = std::min(lo, it->first);
-            hi = std::max(hi, it->first + it->second);
-            it = st->excluded.erase(it);
-        } else {
-            ++it;
-        }
-    }
-    st->excluded.emplace(lo, hi - lo);
+    add_range(st->excluded, a, b);
+    const uint64_t lo = a, hi = b;
     if (st->per_layer == 1) {
         if (st->versions.empty()) {
             layout_slots(st);          // an empty store lays its slots out anew
@@ -2089,15 +2131,35 @@ extern "C" lc_status lc_store_check_dma(lc_store* st, lc_ctx* ctx, uint64_t regi
     std::vector<double> sorted = best;
     std::sort(sorted.begin(), sorted.end());
     const double median = sorted[sorted.size() / 2];
-    uint64_t excluded = 0;
+    // the slow regions, slowest first (lower index first on a tie), each
+    // kept out of use unless that would leave no room for a step that
+    // persists every layer; a store without that room to begin with loses
+    // every slow region
+    std::vector<int64_t> slow;
     for (int64_t i = 0; i < n; ++i) {
         if (rates_out) rates_out[i] = worst[size_t(i)];
-        if (worst[size_t(i)] < min_fraction * median) {
-            const uint64_t off = uint64_t(i) * region_bytes;
-            const uint64_t len = std::min(region_bytes, st->capacity - off);
-            LC_TRY(lc_store_exclude(st, off, len));
-            excluded += len;
-        }
+        if (worst[size_t(i)] < min_fraction * median) slow.push_back(i);
+    }
+    std::stable_sort(slow.begin(), slow.end(),
+                     [&](int64_t a, int64_t b) { return worst[size_t(a)] < worst[size_t(b)]; });
+    const bool guard = full_step_fits(st, st->excluded);
+    RangeMap trial = st->excluded;
+    std::vector<char> take(size_t(n), 0);
+    for (int64_t i : slow) {
+        const uint64_t off = uint64_t(i) * region_bytes;
+        RangeMap next = trial;
+        add_range(next, off, off + std::min(region_bytes, st->capacity - off));
+        if (guard && !full_step_fits(st, next)) continue;
+        trial.swap(next);
+        take[size_t(i)] = 1;
+    }
+    uint64_t excluded = 0;
+    for (int64_t i = 0; i < n; ++i) {
+        if (!take[size_t(i)]) continue;
+        const uint64_t off = uint64_t(i) * region_bytes;
+        const uint64_t len = std::min(region_bytes, st->capacity - off);
+        LC_TRY(lc_store_exclude(st, off, len));
+        excluded += len;
     }
     if (excluded_out) *excluded_out = excluded;
     return LC_OK;

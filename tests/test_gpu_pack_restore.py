@@ -287,34 +287,115 @@ def test_newest_only_store_capacity_and_crash():
     lc.close()
 
 
+def _store_step_sizes(lc, nlayers, per_layer):
+    """Block sizes of a step that persists every layer, in the order an
+    empty store places them: layer order (log store), or each size class,
+    largest first, with one slot per layer of the class plus a spare
+    (newest-only store)."""
+    blocks = [lc.layer_block_bytes(l) for l in range(nlayers)]
+    if per_layer == 0:
+        return blocks
+    rounded = [-(-b // 4096) * 4096 for b in blocks]
+    return [z for z in sorted(set(rounded), reverse=True) for _ in range(rounded.count(z) + 1)]
+
+
+def _fits(sizes, ranges, cap):
+    """Whether blocks of `sizes`, each at the first offset after the previous
+    one that touches none of `ranges`, end within `cap`."""
+    top = 0
+    ranges = sorted(ranges)
+    for z in sizes:
+        at = top
+        for a, n in ranges:
+            if a + n <= at:
+                continue
+            if at + z <= a:
+                break
+            at = a + n
+        if at + z > cap:
+            return False
+        top = at + z
+    return True
+
+
+def _expected_exclusions(rates, fraction, region, cap, sizes):
+    """The regions lc_store_check_dma keeps out of use after one pass (its
+    fastest and slowest pass then coincide): those below fraction x the
+    median rate, slowest first, each unless a full step would then no
+    longer fit (no guard when it did not fit before)."""
+    med = np.sort(rates)[rates.size // 2]
+    slow = sorted((i for i in range(rates.size) if rates[i] < fraction * med), key=lambda i: (rates[i], i))
+    guard = _fits(sizes, [], cap)
+    taken = []
+    for i in slow:
+        r = (i * region, min(region, cap - i * region))
+        if guard and not _fits(sizes, taken + [r], cap):
+            continue
+        taken.append(r)
+    return taken
+
+
+def _full_step(lc, store, t):
+    lc.measure(t)
+    mask, _, _ = lc.select(1e-3, 0)          # staleness bound 0: every layer
+    assert mask.all()
+    lc.pack_async(store)
+    lc.commit_snapshot()
+    lc.wait_durable(t)
+
+
+def _assert_outside(store, ranges):
+    arena = store.info()["arena"]
+    for v in store.versions():
+        off = v["host_ptr"] - arena
+        for h0, hn in ranges:
+            assert off + v["bytes"] <= h0 or off >= h0 + hn, (v, off, h0, hn)
+
+
 def test_store_check_dma_and_exclusions():
-    """lc_store_check_dma times one device->host copy per region of an empty
-    store's arena and excludes the regions below a fraction of the median
-    rate: with fraction 0 nothing goes, with a fraction above 1 exactly the
-    regions below it go (per the rates it reports), with a huge fraction all
-    of them go and a pack finds no room.  Blocks are placed around ranges
-    excluded by lc_store_exclude.  A store holding versions, and a ring
-    store, are refused."""
+    """lc_store_check_dma times device->host copies into every region of an
+    empty store's arena and excludes the slow ones (below a fraction of the
+    median rate), slowest first, while a step that persists every layer
+    still fits.  With fraction 0 nothing goes.  With one pass the excluded
+    regions equal a host-side restatement of that rule over the rates it
+    reports, and a full step then packs around them; with a huge fraction
+    as many regions go as leave room for that step.  A log store too small
+    for a full step loses every region and a pack finds no room.  Blocks
+    are placed around ranges excluded by lc_store_exclude.  A store holding
+    versions, and a ring store, are refused."""
     torch = require_gpu()
     import paper_2609_27193_gb300 as P
     spec = shapes.tiny()
+    N = spec.nlayers
     st = gen.SyntheticState(spec, device="cuda", seed=12)
     lc = make_lc(st, staging_bytes=2 << 20)
-    full = sum(lc.layer_block_bytes(l) for l in range(spec.nlayers))
+    full = sum(lc.layer_block_bytes(l) for l in range(N))
     region = 1 << 20
     t = 0
     for per_layer in (0, 1):
+        sizes = _store_step_sizes(lc, N, per_layer)
         store = P.Store(lc, capacity_bytes=4 * full, versions_per_layer=per_layer)
         cap = store.capacity
         rates, ex = store.check_dma(lc, region_bytes=region, min_fraction=0.0)
         assert ex == 0 and rates.size == -(-cap // region)
         assert np.all(np.isfinite(rates)) and np.all(rates > 0)
-        rates, ex = store.check_dma(lc, region_bytes=region, min_fraction=1.0001, passes=1)
-        med = np.sort(rates)[rates.size // 2]
-        slow = np.flatnonzero(rates < 1.0001 * med)
-        assert ex == sum(min(region, cap - i * region) for i in slow) > 0
-        assert store.info()["excluded_bytes"] == ex
         store.close()
+        for fraction in (1.0001, 1e9):
+            store = P.Store(lc, capacity_bytes=4 * full, versions_per_layer=per_layer)
+            rates, ex = store.check_dma(lc, region_bytes=region, min_fraction=fraction, passes=1)
+            want = _expected_exclusions(rates, fraction, region, cap, sizes)
+            assert ex == sum(n for _, n in want) > 0, (fraction, ex)
+            assert store.info()["excluded_bytes"] == ex
+            if fraction > 1e6:
+                # every region was slow: no further region could go
+                rest = [(i * region, min(region, cap - i * region)) for i in range(rates.size)]
+                rest = [r for r in rest if r not in want]
+                assert rest and not any(_fits(sizes, want + [r], cap) for r in rest)
+            _full_step(lc, store, t)
+            t += 1
+            assert len(store) == N
+            _assert_outside(store, want)
+            store.close()
         # known holes: one inside the base step's stream, one past it
         store = P.Store(lc, capacity_bytes=4 * full, versions_per_layer=per_layer)
         holes = [(full // 2 // 4096 * 4096, 1 << 20), (2 * full // 4096 * 4096, 3 << 20)]
@@ -322,18 +403,11 @@ def test_store_check_dma_and_exclusions():
             store.exclude(*h)
         info = store.info()
         assert info["excluded_bytes"] == sum(h[1] for h in holes)
-        lc.measure(t)
-        lc.select(1e-3, 0)
-        lc.pack_async(store)
-        lc.commit_snapshot()
-        lc.wait_durable(t)
+        _full_step(lc, store, t)
         t += 1
         vers = store.versions()
-        assert len(vers) == spec.nlayers and store.info()["used_bytes"] == full
-        for v in vers:
-            off = v["host_ptr"] - info["arena"]
-            for h0, hn in holes:
-                assert off + v["bytes"] <= h0 or off >= h0 + hn, (v, off, h0)
+        assert len(vers) == N and store.info()["used_bytes"] == full
+        _assert_outside(store, holes)
         with pytest.raises(P.LCError) as e:
             store.check_dma(lc, region_bytes=region)
         assert e.value.status == 2
@@ -341,18 +415,19 @@ def test_store_check_dma_and_exclusions():
             store.exclude(vers[0]["host_ptr"] - info["arena"], 4096)     # a block lies there
         assert e.value.status == 2
         store.close()
-        empty = P.Store(lc, capacity_bytes=4 * full, versions_per_layer=per_layer)
-        empty.check_dma(lc, region_bytes=region, min_fraction=1e9)     # every region excluded
-        assert empty.info()["excluded_bytes"] == empty.capacity
-        lc.measure(t)
-        lc.select(1e-3, 0)
-        t += 1
-        with pytest.raises(P.LCError) as e:
-            lc.pack_async(empty)
-        assert e.value.status == 5
-        lc.pack_device(torch.empty(full, dtype=torch.uint8, device="cuda"))
-        lc.commit_snapshot()
-        empty.close()
+    # a log store that cannot take a full step: no guard, every region goes
+    small = P.Store(lc, capacity_bytes=full // 2)
+    small.check_dma(lc, region_bytes=region, min_fraction=1e9)
+    assert small.info()["excluded_bytes"] == small.capacity
+    lc.measure(t)
+    lc.select(1e-3, 0)
+    t += 1
+    with pytest.raises(P.LCError) as e:
+        lc.pack_async(small)
+    assert e.value.status == 5
+    lc.pack_device(torch.empty(full, dtype=torch.uint8, device="cuda"))
+    lc.commit_snapshot()
+    small.close()
     ring = P.Store(lc, versions_per_layer=2)
     with pytest.raises(P.LCError) as e:
         ring.exclude(0, 4096)
