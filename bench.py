@@ -75,6 +75,10 @@ def parse_args():
     ap.add_argument("--no-configs", action="store_true",
                     help="skip the short passes over the other workloads (tiny, 1b, 8b at tau 5e-4 "
                          "and 2e-3, 8b-tensor, 8b-cadence) that the default 8b run adds as `configs`")
+    ap.add_argument("--host-store-gb", type=float, default=0.0,
+                    help="cap the pinned store of the e2e leg (GB; 0: 1.25 x the full state, at most 60%% of "
+                         "the host's available memory per local rank); steps that do not fit then pack "
+                         "into device memory and are left out of e2e")
     ap.add_argument("--no-dma-check", action="store_true",
                     help="do not run lc_store_check_dma on the e2e store (by default the pinned "
                          "regions the GPU copies into at under half the median rate are kept out of use)")
@@ -714,6 +718,7 @@ def run_ours(args):
 
     graph = args.path == "graph"
     overflow = []
+    spill_ok = [False]      # e2e: the host store cannot take a full step
 
     def graph_step(t, ev, h0):
         ev[0].record(side)
@@ -763,7 +768,15 @@ def run_ours(args):
         if mode == "device":
             lc.pack_device(dst)
         else:
-            lc.pack_async(store)
+            try:
+                lc.pack_async(store)
+            except P.LCError as err:
+                # a store smaller than a full step: this step's layers go to
+                # device memory instead, and the step is left out of e2e
+                if err.status != 5 or not spill_ok[0]:
+                    raise
+                lc.pack_device(dst)
+                mode = "spilled"
         ev[3].record(side)
         lc.commit_snapshot()
         ev[4].record(side)
@@ -771,7 +784,8 @@ def run_ours(args):
             lc.wait_durable(t)
         h2 = time.perf_counter()
         main.wait_stream(side)
-        return dict(ev=ev, decision_s=h1 - h0, host_s=h2 - h0, mask=mask, nbytes=nbytes)
+        return dict(ev=ev, decision_s=h1 - h0, host_s=h2 - h0, mask=mask, nbytes=nbytes,
+                    spilled=mode == "spilled")
 
     if graph:
         lc.step_graph_create(tau, K, dst)
@@ -890,6 +904,8 @@ def run_ours(args):
                         avail = int(line.split()[1]) * 1024
         except OSError:
             pass
+        # ranks on one host share its memory: each pins at most its share
+        avail //= max(1, int(os.environ.get("LOCAL_WORLD_SIZE", world)))
         dma_check = None
         if graph:
             # the replayed pack writes straight into pinned host memory
@@ -901,6 +917,9 @@ def run_ours(args):
             # a quarter of the full state as headroom for regions the DMA
             # check keeps out of use (pinned pages the GPU reaches slowly)
             cap = int(full * 1.25) if avail == 0 else min(int(full * 1.25), int(avail * 0.6))
+            if args.host_store_gb > 0:
+                cap = min(cap, int(args.host_store_gb * 1e9))
+            spill_ok[0] = cap < full
             store = P.Store(lc, capacity_bytes=cap)
             if not args.no_dma_check:
                 region = 256 << 20
@@ -928,6 +947,7 @@ def run_ours(args):
                 files_note = ("skipped: about %.0f GB would be written, %.0f GB free on %s"
                               % (need / 1e9, free / 1e9, args.files))
         traces = []
+        spilled = 0
         for i in range(max(1, args.warmup) + args.steps):
             t += 1
             if store is not None:
@@ -948,16 +968,33 @@ def run_ours(args):
             if store is not None:
                 store.clear()
             if i >= max(1, args.warmup):
+                if r.get("spilled"):
+                    spilled += 1
+                    continue
                 e_recs.append(r)
                 e_bytes.append(mbytes + pack_bytes(r["mask"], payload, wbytes, fused_commit=pack_commit))
         if store is not None:
             lc.trace_copies(False)
         link_after = d2h_link_probe(torch, dev)
         e_s = sum(r["host_s"] for r in e_recs)
+        e_tot = float(sum(e_bytes))
+        if not e_recs:
+            raise SystemExit("bench: every timed e2e step persisted more than the %.1f GB host store holds "
+                             "(--host-store-gb)" % (cap / 1e9))
         d2h = statistics.mean(r["nbytes"] for r in e_recs)
-        e2e = {"value": sum(e_bytes) / e_s / 1e9, "unit": "GB/s", "h2d_bytes_per_step": 0,
+        if world > 1:
+            # whole job: every rank's bytes over the slowest rank's time
+            tb = torch.tensor([e_tot], dtype=torch.float64, device=dev)
+            tt = torch.tensor([e_s], dtype=torch.float64, device=dev)
+            dist.all_reduce(tb)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            e_tot, e_s = tb.item(), tt.item()
+        e2e = {"value": e_tot / e_s / 1e9, "unit": "GB/s", "h2d_bytes_per_step": 0,
                "d2h_bytes_per_step": int(d2h),
                "ms_per_step": 1e3 * e_s / len(e_recs),
+               # steps whose layers did not fit a store smaller than a full step
+               # (--host-store-gb, or a host without room for one per rank)
+               "steps_spilled_to_device": spilled,
                "d2h_GBps": d2h / (statistics.mean((r["host_s"] - r["decision_s"]) if not graph
                                                   else r["host_s"] for r in e_recs)) / 1e9,
                # the host link and host memory are shared with other jobs on the
