@@ -476,6 +476,29 @@ def d2h_link_probe(torch, dev, nbytes=4 << 30):
     return best
 
 
+def d2h_streams_probe(torch, dev, nbytes=4 << 30, chunk=256 << 20):
+    """The same copy split into chunks spread round-robin over 1, 2 and 4
+    streams (best of 3 each): whether concurrent copies get more of the
+    host link than one."""
+    d = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    h = torch.empty(nbytes, dtype=torch.uint8, pin_memory=True)
+    out = {}
+    for ns in (1, 2, 4):
+        streams = [torch.cuda.Stream(device=dev) for _ in range(ns)]
+        best = 0.0
+        for _ in range(3):
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            for i in range(nbytes // chunk):
+                with torch.cuda.stream(streams[i % ns]):
+                    h[i * chunk:(i + 1) * chunk].copy_(d[i * chunk:(i + 1) * chunk], non_blocking=True)
+            torch.cuda.synchronize()
+            best = max(best, nbytes / (time.perf_counter() - t0) / 1e9)
+        out[str(ns)] = round(best, 1)
+    del d, h
+    return out
+
+
 def config_pass(P, torch, dev, st, units, nunits, tau, K, steps, warmup, scales_for, dst, hbm,
                 per_tensor=False, gemm=None, regime_of=None, l2_bytes=128 << 20):
     """One short device-resident pass over a workload: a fresh context whose
@@ -976,6 +999,7 @@ def run_ours(args):
         if store is not None:
             lc.trace_copies(False)
         link_after = d2h_link_probe(torch, dev)
+        link_streams = d2h_streams_probe(torch, dev)
         e_s = sum(r["host_s"] for r in e_recs)
         e_tot = float(sum(e_bytes))
         if not e_recs:
@@ -1003,6 +1027,9 @@ def run_ours(args):
                "d2h_link_GBps_measured": link,
                "store_dma_check": dma_check,
                "d2h_link_GBps_after": link_after,
+               # GB/s by number of concurrent copy streams: the link, not the
+               # number of copy engines in use, sets the rate
+               "d2h_link_GBps_by_streams": link_streams,
                "steps_d2h_ms": [round(1e3 * ((r["host_s"] - r["decision_s"]) if not graph else r["host_s"]), 3)
                                 for r in e_recs],
                "steps_d2h_bytes": [int(r["nbytes"]) for r in e_recs],
