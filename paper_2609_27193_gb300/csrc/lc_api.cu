@@ -1373,6 +1373,23 @@ extern "C" lc_status lc_pack_async(lc_ctx* ctx, lc_store* st) {
                            st->versions.end());
         return LC_OK;
     };
+    // If an error ends the loop below after copies into the arena were
+    // enqueued, the store still learns when they are done, so that it is
+    // not freed or cleared under them.
+    struct InflightGuard {
+        lc_store* st;
+        cudaStream_t s;
+        bool armed = false;
+        ~InflightGuard() {
+            if (!armed) return;
+            cudaEvent_t ev = nullptr;
+            if (cudaEventCreateWithFlags(&ev, cudaEventDisableTiming) == cudaSuccess) {
+                if (cudaEventRecord(ev, s) == cudaSuccess) st->inflight.push_back(ev);
+                else cudaEventDestroy(ev);
+            }
+            cudaGetLastError();
+        }
+    } guard{st, ctx->copy_stream};
     // ring: gather chunk c into slot c%2 on the stream, copy it out on the copy stream
     const uint64_t S = ctx->slot_bytes;
     for (uint64_t lo = 0, c = 0; lo < bytes; lo += S, ++c) {
@@ -1402,6 +1419,7 @@ extern "C" lc_status lc_pack_async(lc_ctx* ctx, lc_store* st) {
                     }
                 }
             }
+            guard.armed = true;
             LC_CUDA(cudaMemcpyAsync(e.host + (a - e.soff), slot + (a - lo), b - a, cudaMemcpyDeviceToHost,
                                     ctx->copy_stream));
             ctx->counters.d2h_bytes += b - a;
@@ -1423,12 +1441,19 @@ extern "C" lc_status lc_pack_async(lc_ctx* ctx, lc_store* st) {
     PendingPack pp;
     pp.step = ctx->hdr.step;
     pp.store = st;
-    LC_CUDA(cudaEventCreateWithFlags(&pp.done, cudaEventDisableTiming));
-    LC_CUDA(cudaEventRecord(pp.done, ctx->copy_stream));
     cudaEvent_t inflight;
     LC_CUDA(cudaEventCreateWithFlags(&inflight, cudaEventDisableTiming));
-    LC_CUDA(cudaEventRecord(inflight, ctx->copy_stream));
+    if (cudaEventRecord(inflight, ctx->copy_stream) != cudaSuccess) {
+        cudaEventDestroy(inflight);
+        LC_CUDA(cudaGetLastError());
+    }
     st->inflight.push_back(inflight);
+    guard.armed = false;   // the store tracks the copies from here on
+    LC_CUDA(cudaEventCreateWithFlags(&pp.done, cudaEventDisableTiming));
+    if (cudaEventRecord(pp.done, ctx->copy_stream) != cudaSuccess) {
+        cudaEventDestroy(pp.done);
+        LC_CUDA(cudaGetLastError());
+    }
     for (const StoreVersion& v : fresh) {
         st->versions.push_back(v);
         pp.ids.push_back(v.id);
