@@ -455,6 +455,7 @@ typedef struct {
     uint64_t used_bytes;       /* bytes held by versions, pending or durable    */
     int32_t versions_per_layer;
     int32_t reserved;
+    uint64_t avoided_bytes;    /* slow bytes left in use by lc_store_check_dma  */
 } lc_store_info;
 
 /* Errors: INVALID_ARG (NULL). */
@@ -484,8 +485,12 @@ lc_status lc_store_exclude(lc_store* store, uint64_t offset, uint64_t bytes);
  * stays in use: every layer's block in layer order from offset 0 (log
  * store), or each block size's slots for its layers plus the spare
  * (newest-only store).  A store that lacks that room before the call loses
- * every slow region.  region_bytes: 0 (256 MiB) or a multiple of 4096 in
- * [1 MiB, 1 GiB]; passes: 0 (4) or 1..64.
+ * every slow region.  The slow regions left in use are avoided: a log store
+ * places a step's blocks off them whenever the whole step fits that way,
+ * and a newest-only store lays its slots out off them whenever its layers'
+ * slots and spares fit that way (lc_store_info.avoided_bytes); each call
+ * replaces the previous call's avoided regions.  region_bytes: 0 (256 MiB)
+ * or a multiple of 4096 in [1 MiB, 1 GiB]; passes: 0 (4) or 1..64.
  * rates_out (host, nullable): each of the ceil(capacity / region_bytes)
  * regions' slowest GB/s; excluded_out (nullable): bytes excluded.
  * Overwrites the arena; blocks (bounded by ctx's timeout_ms).

@@ -379,7 +379,8 @@ class Store:
         i = lc_store_info()
         check(self._lib.lc_store_get_info(self._h, C.byref(i)))
         return dict(arena=i.arena, capacity=i.capacity, excluded_bytes=i.excluded_bytes,
-                    used_bytes=i.used_bytes, versions_per_layer=i.versions_per_layer)
+                    used_bytes=i.used_bytes, versions_per_layer=i.versions_per_layer,
+                    avoided_bytes=i.avoided_bytes)
 
     @property
     def capacity(self):

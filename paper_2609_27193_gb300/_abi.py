@@ -78,7 +78,8 @@ class lc_manifest_record(C.Structure):
 
 class lc_store_info(C.Structure):
     _fields_ = [("arena", C.c_void_p), ("capacity", C.c_uint64), ("excluded_bytes", C.c_uint64),
-                ("used_bytes", C.c_uint64), ("versions_per_layer", C.c_int32), ("reserved", C.c_int32)]
+                ("used_bytes", C.c_uint64), ("versions_per_layer", C.c_int32), ("reserved", C.c_int32),
+                ("avoided_bytes", C.c_uint64)]
 
 
 class lc_copy_span(C.Structure):

@@ -159,6 +159,9 @@ struct lc_store {
     std::vector<uint64_t> layer_base;      // ring mode
     std::vector<int64_t> layer_writes;     // ring mode: versions ever written
     std::map<uint64_t, uint64_t> excluded; // ranges kept out of use (lc_store_exclude), disjoint
+    // slow regions that lc_store_check_dma left in use to keep room for a
+    // full step: a placement uses them only when it does not fit without them
+    std::map<uint64_t, uint64_t> avoid;
     // newest-only mode: layers whose blocks have the same size share a class
     // of slots (its layers' slots plus spares); a free slot list per class
     std::vector<int32_t> layer_class;
@@ -220,6 +223,13 @@ std::vector<size_t> classes_largest_first(const lc_store* st) {
     return order;
 }
 
+// The excluded ranges together with the ranges to avoid.
+RangeMap excluded_and_avoided(const lc_store* st) {
+    RangeMap m = st->excluded;
+    for (const auto& x : st->avoid) add_range(m, x.first, x.first + x.second);
+    return m;
+}
+
 // Whether the store, empty and with `excl` out of use, takes a step that
 // persists every layer: in a log store every layer's block in layer order
 // from offset 0; in a newest-only store each size class's slots for its
@@ -245,16 +255,20 @@ bool full_step_fits(const lc_store* st, const RangeMap& excl) {
 
 // Newest-only mode: lays the slots out in an empty store, skipping excluded
 // ranges -- classes largest first, each its layers' slots plus one spare,
-// then further spares class by class while they fit.
+// then further spares class by class while they fit.  The slots keep off
+// the ranges to avoid too, unless the layers' slots and spares then do not
+// fit.
 void layout_slots(lc_store* st) {
     const size_t nc = st->class_bytes.size();
     const std::vector<size_t> order = classes_largest_first(st);
+    const RangeMap both = excluded_and_avoided(st);
+    const RangeMap& keep_off = !st->avoid.empty() && full_step_fits(st, both) ? both : st->excluded;
     st->class_slots.assign(nc, 0);
     st->class_free.assign(nc, {});
     uint64_t top = 0;
     auto place = [&](size_t c) -> bool {
         const uint64_t z = st->class_bytes[c];
-        const uint64_t at = log_place(st, top, z);
+        const uint64_t at = place_around(keep_off, top, z);
         if (at + z > st->capacity) return false;
         st->class_free[c].push_back(at);
         st->class_slots[c] += 1;
@@ -1260,16 +1274,29 @@ extern "C" lc_status lc_pack_async(lc_ctx* ctx, lc_store* st) {
     std::vector<std::vector<int32_t>> wait_before;   // newest-only: layers to see complete first
     if (st->per_layer == 0) {
         // each layer block goes to the next offset that touches no excluded
-        // range; blocks that land back to back share one extent
+        // range, and no range to avoid unless the step does not fit that
+        // way; blocks that land back to back share one extent
+        std::vector<uint64_t> at_of(size_t(ctx->nlayers), 0);
+        auto place_step = [&](const RangeMap& keep_off) -> bool {
+            uint64_t c = st->top;
+            for (int32_t l = 0; l < ctx->nlayers; ++l) {
+                if (!ctx->mask[l]) continue;
+                const uint64_t lb = ctx->layer_bytes[l];
+                const uint64_t at = place_around(keep_off, c, lb);
+                if (at + lb > st->capacity) return false;
+                at_of[size_t(l)] = at;
+                c = at + lb;
+            }
+            return true;
+        };
+        if (!(!st->avoid.empty() && place_step(excluded_and_avoided(st))) && !place_step(st->excluded))
+            return fail(LC_ERR_CAPACITY, "lc_pack_async: store holds %llu of %llu bytes, %llu more needed",
+                        (unsigned long long)st->top, (unsigned long long)st->capacity, (unsigned long long)bytes);
         uint64_t cur = st->top;
         for (int32_t l = 0; l < ctx->nlayers; ++l) {
             if (!ctx->mask[l]) continue;
             const uint64_t lb = ctx->layer_bytes[l];
-            const uint64_t at = log_place(st, cur, lb);
-            if (at + lb > st->capacity)
-                return fail(LC_ERR_CAPACITY, "lc_pack_async: store holds %llu of %llu bytes, %llu more needed",
-                            (unsigned long long)st->top, (unsigned long long)st->capacity,
-                            (unsigned long long)bytes);
+            const uint64_t at = at_of[size_t(l)];
             uint8_t* host = st->arena + at;
             if (!ext.empty() && ext.back().soff + ext.back().len == ctx->offsets[l] &&
                 ext.back().host + ext.back().len == host)
@@ -2012,6 +2039,7 @@ extern "C" lc_status lc_store_get_info(const lc_store* st, lc_store_info* out) {
     out->arena = st->arena;
     out->capacity = st->capacity;
     for (const auto& x : st->excluded) out->excluded_bytes += x.second;
+    for (const auto& x : st->avoid) out->avoided_bytes += x.second;
     for (const StoreVersion& v : st->versions) out->used_bytes += v.bytes;
     out->versions_per_layer = st->per_layer;
     return LC_OK;
@@ -2178,6 +2206,14 @@ extern "C" lc_status lc_store_check_dma(lc_store* st, lc_ctx* ctx, uint64_t regi
         trial.swap(next);
         take[size_t(i)] = 1;
     }
+    // the slow regions left in use are avoided while a step fits without them
+    RangeMap avoid;
+    for (int64_t i : slow) {
+        if (take[size_t(i)]) continue;
+        const uint64_t off = uint64_t(i) * region_bytes;
+        add_range(avoid, off, off + std::min(region_bytes, st->capacity - off));
+    }
+    st->avoid.swap(avoid);
     uint64_t excluded = 0;
     for (int64_t i = 0; i < n; ++i) {
         if (!take[size_t(i)]) continue;
@@ -2186,6 +2222,7 @@ extern "C" lc_status lc_store_check_dma(lc_store* st, lc_ctx* ctx, uint64_t regi
         LC_TRY(lc_store_exclude(st, off, len));
         excluded += len;
     }
+    if (st->per_layer == 1 && excluded == 0) layout_slots(st);   // with the new ranges to avoid
     if (excluded_out) *excluded_out = excluded;
     return LC_OK;
 }

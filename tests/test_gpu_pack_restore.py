@@ -322,17 +322,19 @@ def _expected_exclusions(rates, fraction, region, cap, sizes):
     """The regions lc_store_check_dma keeps out of use after one pass (its
     fastest and slowest pass then coincide): those below fraction x the
     median rate, slowest first, each unless a full step would then no
-    longer fit (no guard when it did not fit before)."""
+    longer fit (no guard when it did not fit before).  Returns those and the
+    slow regions left in use (to be avoided)."""
     med = np.sort(rates)[rates.size // 2]
     slow = sorted((i for i in range(rates.size) if rates[i] < fraction * med), key=lambda i: (rates[i], i))
     guard = _fits(sizes, [], cap)
-    taken = []
+    taken, kept = [], []
     for i in slow:
         r = (i * region, min(region, cap - i * region))
         if guard and not _fits(sizes, taken + [r], cap):
+            kept.append(r)
             continue
         taken.append(r)
-    return taken
+    return taken, kept
 
 
 def _full_step(lc, store, t):
@@ -356,10 +358,13 @@ def test_store_check_dma_and_exclusions():
     """lc_store_check_dma times device->host copies into every region of an
     empty store's arena and excludes the slow ones (below a fraction of the
     median rate), slowest first, while a step that persists every layer
-    still fits.  With fraction 0 nothing goes.  With one pass the excluded
-    regions equal a host-side restatement of that rule over the rates it
-    reports, and a full step then packs around them; with a huge fraction
-    as many regions go as leave room for that step.  A log store too small
+    still fits; the slow regions left in use are avoided by every placement
+    that fits without them.  With fraction 0 nothing goes.  With one pass
+    the excluded and avoided regions equal a host-side restatement of that
+    rule over the rates it reports, a full step then packs around the
+    excluded ones (and the avoided ones if it fits so), and a one-layer
+    step of the log store keeps off both; with a huge fraction as many
+    regions go as leave room for that step.  A log store too small
     for a full step loses every region and a pack finds no room.  Blocks
     are placed around ranges excluded by lc_store_exclude.  A store holding
     versions, and a ring store, are refused."""
@@ -383,9 +388,10 @@ def test_store_check_dma_and_exclusions():
         for fraction in (1.0001, 1e9):
             store = P.Store(lc, capacity_bytes=4 * full, versions_per_layer=per_layer)
             rates, ex = store.check_dma(lc, region_bytes=region, min_fraction=fraction, passes=1)
-            want = _expected_exclusions(rates, fraction, region, cap, sizes)
+            want, kept = _expected_exclusions(rates, fraction, region, cap, sizes)
             assert ex == sum(n for _, n in want) > 0, (fraction, ex)
             assert store.info()["excluded_bytes"] == ex
+            assert store.info()["avoided_bytes"] == sum(n for _, n in kept)
             if fraction > 1e6:
                 # every region was slow: no further region could go
                 rest = [(i * region, min(region, cap - i * region)) for i in range(rates.size)]
@@ -395,6 +401,24 @@ def test_store_check_dma_and_exclusions():
             t += 1
             assert len(store) == N
             _assert_outside(store, want)
+            if _fits(sizes, want + kept, cap):
+                _assert_outside(store, kept)
+            if per_layer == 0 and kept:
+                # one layer's block keeps off the slow regions left in use
+                store.clear()
+                scales = np.zeros(N)
+                scales[1] = 1e-2
+                st.drift(1000 + t, scales)
+                lc.measure(t)
+                mask, _, _ = lc.select(1e-12, 1 << 20)
+                assert mask.tolist() == [int(l == 1) for l in range(N)]
+                lc.pack_async(store)
+                lc.commit_snapshot()
+                lc.wait_durable(t)
+                t += 1
+                assert len(store) == 1
+                if _fits([lc.layer_block_bytes(1)], want + kept, cap):
+                    _assert_outside(store, want + kept)
             store.close()
         # known holes: one inside the base step's stream, one past it
         store = P.Store(lc, capacity_bytes=4 * full, versions_per_layer=per_layer)
