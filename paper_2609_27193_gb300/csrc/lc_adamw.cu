@@ -527,7 +527,8 @@ __global__ void __launch_bounds__(kMeasureThreads, 1) adamw_bulk_kernel(const Me
     __syncthreads();
     if (s_ticket != gridDim.x - 1) return;
     __threadfence();
-    finalize(p);
+    // every load and bulk store of the ring is complete: it stages the combine
+    finalize(p, reinterpret_cast<double2*>(ring), int32_t(kAdamBulkSmem / sizeof(double2)));
 }
 
 }  // namespace

@@ -425,7 +425,8 @@ __global__ void __launch_bounds__(kMeasureThreads, 1) measure_bulk_kernel(const 
     __syncthreads();
     if (s_ticket != gridDim.x - 1) return;
     __threadfence();
-    finalize(p);
+    // the ring's loads have all landed (or the CTA gave up): it stages the combine
+    finalize(p, reinterpret_cast<double2*>(ring), int32_t(kMeasureBulkSmem / sizeof(double2)));
 }
 
 }  // namespace
