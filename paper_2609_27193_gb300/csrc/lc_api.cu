@@ -808,6 +808,7 @@ static lc_status register_layout_impl(lc_ctx* ctx, const lc_segment* segs, int32
     ctx->layer_bytes.assign(nlayers, 0);
     ctx->layer_sec_begin.assign(nlayers + 1, 0);
     std::vector<int32_t> wsec(nlayers, 0);
+    std::vector<uint64_t> commit_work(nlayers, 0);
     ctx->secs.clear();
     ctx->sec_seg.clear();
     ctx->sec_part.clear();
@@ -830,6 +831,10 @@ static lc_status register_layout_impl(lc_ctx* ctx, const lc_segment* segs, int32
                           : part == 1 ? reinterpret_cast<const uint8_t*>(sg.exp_avg)
                                       : reinterpret_cast<const uint8_t*>(sg.exp_avg_sq);
                 sec.ref = part == 0 ? static_cast<uint8_t*>(sg.snap) : nullptr;
+                sec.commit_off = part == 0 ? commit_work[l] : 0;
+                sec.layer = l;
+                sec.idx = int32_t(ctx->secs.size()) - ctx->layer_sec_begin[l];
+                if (part == 0) commit_work[l] += round_up(nbytes, 16);
                 ctx->secs.push_back(sec);
                 ctx->sec_seg.push_back(i);
                 ctx->sec_part.push_back(part);
@@ -871,6 +876,7 @@ static lc_status register_layout_impl(lc_ctx* ctx, const lc_segment* segs, int32
     const size_t o_lbytes = tp.take(sizeof(uint64_t) * nlayers);
     const size_t o_lsec = tp.take(sizeof(int32_t) * (nlayers + 1));
     const size_t o_lwsec = tp.take(sizeof(int32_t) * nlayers);
+    const size_t o_lcw = tp.take(sizeof(uint64_t) * nlayers);
     const size_t o_secs = tp.take(sizeof(SectionDev) * std::max(1, nsec));
     const size_t o_scratch = tp.take(sizeof(int64_t) * 3 * nlayers);
     const size_t o_accsave = tp.take(sizeof(double) * nlayers);
@@ -904,6 +910,7 @@ static lc_status register_layout_impl(lc_ctx* ctx, const lc_segment* segs, int32
     put(o_lbytes, ctx->layer_bytes.data(), sizeof(uint64_t) * nlayers);
     put(o_lsec, ctx->layer_sec_begin.data(), sizeof(int32_t) * (nlayers + 1));
     put(o_lwsec, wsec.data(), sizeof(int32_t) * nlayers);
+    put(o_lcw, commit_work.data(), sizeof(uint64_t) * nlayers);
     put(o_secs, ctx->secs.data(), sizeof(SectionDev) * nsec);
     // accumulators, t_l, ticket and partials start at zero (the host image is zeroed)
 
@@ -948,6 +955,7 @@ static lc_status register_layout_impl(lc_ctx* ctx, const lc_segment* segs, int32
     sp.layer_bytes = reinterpret_cast<const uint64_t*>(base + o_lbytes);
     sp.layer_sec_begin = reinterpret_cast<const int32_t*>(base + o_lsec);
     sp.layer_wsec_count = reinterpret_cast<const int32_t*>(base + o_lwsec);
+    sp.layer_commit_work = reinterpret_cast<const uint64_t*>(base + o_lcw);
     sp.secs = reinterpret_cast<const SectionDev*>(base + o_secs);
     sp.layer_scratch = reinterpret_cast<int64_t*>(base + o_scratch);
     sp.acc_save = reinterpret_cast<double*>(base + o_accsave);

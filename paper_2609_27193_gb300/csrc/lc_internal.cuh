@@ -107,6 +107,9 @@ struct SectionDev {
     uint64_t span;
     const uint8_t* src;
     uint8_t* ref;         // snapshot of a W section (for the fused commit), else null
+    uint64_t commit_off;  // W section: its offset in the layer's commit work space
+    int32_t layer;
+    int32_t idx;          // position among the layer's sections
 };
 
 // Layout of the decision block written by the select kernel and mirrored
@@ -151,6 +154,7 @@ struct SelectParams {
     const uint64_t* layer_bytes;     // [nlayers] packed block bytes
     const int32_t* layer_sec_begin;  // [nlayers+1] sections of layer l (packed order)
     const int32_t* layer_wsec_count; // [nlayers] W sections of layer l (first in its range)
+    const uint64_t* layer_commit_work; // [nlayers] commit work bytes of layer l's W sections
     const SectionDev* secs;
     int64_t* layer_scratch;          // [3*nlayers] per-layer output indices
     uint8_t* result;                 // decision block (device)

@@ -83,10 +83,9 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectPara
             uint64_t cw = 0;
             int ns = 0, nw = 0;
             if (sel) {
-                const int s0 = p.layer_sec_begin[l];
-                ns = p.layer_sec_begin[l + 1] - s0;
+                ns = p.layer_sec_begin[l + 1] - p.layer_sec_begin[l];
                 nw = p.layer_wsec_count[l];
-                for (int j = s0; j < s0 + nw; ++j) cw += (p.secs[j].nbytes + 15) & ~uint64_t(15);
+                cw = p.layer_commit_work[l];
             }
             t_bytes[threadIdx.x] = sel ? p.layer_bytes[l] : 0;
             t_cw[threadIdx.x] = cw;
@@ -146,35 +145,32 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectPara
         }
         return;
     }
+    // the copy lists, one section per thread: a persisted layer's sections
+    // go to its pack entries (and its W sections to its commit entries) at
+    // the indices and offsets laid out above
     const bool fused = p.fuse_commit != 0 && p.mode == 0;
-    for (int l = threadIdx.x; l < p.nlayers; l += blockDim.x) {
+    const int nsec_all = p.layer_sec_begin[p.nlayers];
+    for (int j = threadIdx.x; j < nsec_all; j += blockDim.x) {
+        const SectionDev sec = p.secs[j];
+        const int l = sec.layer;
         if (!mask[l]) continue;
-        const int s0 = p.layer_sec_begin[l], s1 = p.layer_sec_begin[l + 1];
-        int64_t di = scratch[3 * l];
-        for (int j = s0; j < s1; ++j, ++di) {
-            const SectionDev sec = p.secs[j];
-            CopyDesc d;
-            d.woff = off[l] + sec.off_in_layer;
-            d.nbytes = sec.nbytes;
-            d.span = sec.span;
-            d.src = sec.src;
-            d.dst = nullptr;
-            d.dst2 = (fused && sec.ref) ? sec.ref : nullptr;
-            p.pack_desc[di] = d;
-        }
-        int64_t ci = scratch[3 * l + 1];
-        uint64_t cw = uint64_t(scratch[3 * l + 2]);
-        for (int j = s0; j < s0 + p.layer_wsec_count[l]; ++j, ++ci) {
-            const SectionDev sec = p.secs[j];
-            CopyDesc d;
-            d.woff = cw;
-            d.nbytes = sec.nbytes;
-            d.span = (sec.nbytes + 15) & ~uint64_t(15);
-            d.src = sec.src;
-            d.dst = sec.ref;
-            d.dst2 = nullptr;
-            p.commit_desc[ci] = d;
-            cw += d.span;
+        CopyDesc d;
+        d.woff = off[l] + sec.off_in_layer;
+        d.nbytes = sec.nbytes;
+        d.span = sec.span;
+        d.src = sec.src;
+        d.dst = nullptr;
+        d.dst2 = (fused && sec.ref) ? sec.ref : nullptr;
+        p.pack_desc[scratch[3 * l] + sec.idx] = d;
+        if (sec.idx < p.layer_wsec_count[l]) {
+            CopyDesc c;
+            c.woff = uint64_t(scratch[3 * l + 2]) + sec.commit_off;
+            c.nbytes = sec.nbytes;
+            c.span = (sec.nbytes + 15) & ~uint64_t(15);
+            c.src = sec.src;
+            c.dst = sec.ref;
+            c.dst2 = nullptr;
+            p.commit_desc[scratch[3 * l + 1] + sec.idx] = c;
         }
     }
 }
