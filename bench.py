@@ -94,6 +94,21 @@ def dist_env():
     return rank, world, local
 
 
+def whole_job(nbytes, seconds, world, device):
+    """(bytes, seconds) of the whole job: every rank's bytes over the slowest
+    rank's time, so that bytes / seconds is the job's rate (weak scaling:
+    each rank moves its own bytes).  One rank: the inputs unchanged."""
+    if world <= 1:
+        return float(nbytes), float(seconds)
+    import torch
+    import torch.distributed as dist
+    tb = torch.tensor([float(nbytes)], dtype=torch.float64, device=device)
+    tt = torch.tensor([float(seconds)], dtype=torch.float64, device=device)
+    dist.all_reduce(tb)
+    dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+    return tb.item(), tt.item()
+
+
 def peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -847,12 +862,7 @@ def run_ours(args):
     tot_bytes = sum(mbytes + pb for pb in pbytes)
     tot_s = sum(step_ms) / 1e3
     frac_sel = float(np.mean([r["mask"].mean() for r in recs]))
-    if world > 1:
-        tb = torch.tensor([float(tot_bytes)], device=dev)
-        tt = torch.tensor([tot_s], device=dev)
-        dist.all_reduce(tb)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        tot_bytes, tot_s = tb.item(), tt.item()
+    tot_bytes, tot_s = whole_job(tot_bytes, tot_s, world, dev)
     value = tot_bytes / tot_s / 1e9
     regimes = None
     if wl.regimes:
@@ -1008,13 +1018,7 @@ def run_ours(args):
             raise SystemExit("bench: every timed e2e step persisted more than the %.1f GB host store holds "
                              "(--host-store-gb)" % (cap / 1e9))
         d2h = statistics.mean(r["nbytes"] for r in e_recs)
-        if world > 1:
-            # whole job: every rank's bytes over the slowest rank's time
-            tb = torch.tensor([e_tot], dtype=torch.float64, device=dev)
-            tt = torch.tensor([e_s], dtype=torch.float64, device=dev)
-            dist.all_reduce(tb)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            e_tot, e_s = tb.item(), tt.item()
+        e_tot, e_s = whole_job(e_tot, e_s, world, dev)
         e2e = {"value": e_tot / e_s / 1e9, "unit": "GB/s", "h2d_bytes_per_step": 0,
                "d2h_bytes_per_step": int(d2h),
                "ms_per_step": 1e3 * e_s / len(e_recs),
