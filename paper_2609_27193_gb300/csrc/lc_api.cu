@@ -179,17 +179,35 @@ namespace {
 // Blocks of a newest-only store start on this boundary.
 constexpr uint64_t kStoreGrain = 4096;
 
-using RangeMap = std::map<uint64_t, uint64_t>;   // offset -> length, disjoint
+using RangeMap = std::map<uint64_t, uint64_t>;   // offset -> length, disjoint ranges
 
 // The first offset >= `from` at which `len` bytes touch no range of `excl`.
+// Only the last range beginning at or before `from` can contain it; the
+// ranges after it are passed over while the block runs into them.
 uint64_t place_around(const RangeMap& excl, uint64_t from, uint64_t len) {
     uint64_t at = from;
-    for (const auto& x : excl) {
-        if (x.first + x.second <= at) continue;
-        if (at + len <= x.first) break;
-        at = x.first + x.second;
+    auto it = excl.upper_bound(at);
+    if (it != excl.begin()) {
+        auto prev = std::prev(it);
+        if (prev->first + prev->second > at) it = prev;
+    }
+    for (; it != excl.end(); ++it) {
+        if (at + len <= it->first) break;
+        at = it->first + it->second;
     }
     return at;
+}
+
+// The same for the union of two maps (each disjoint, possibly overlapping
+// each other): alternate until neither moves the block.
+uint64_t place_around(const RangeMap& a, const RangeMap& b, uint64_t from, uint64_t len) {
+    uint64_t at = from;
+    for (;;) {
+        const uint64_t x = place_around(a, at, len);
+        const uint64_t y = place_around(b, x, len);
+        if (y == x) return x;
+        at = y;
+    }
 }
 
 // Log mode: the first offset >= `from` at which `len` bytes touch no
@@ -230,14 +248,15 @@ RangeMap excluded_and_avoided(const lc_store* st) {
     return m;
 }
 
-// Whether the store, empty and with `excl` out of use, takes a step that
-// persists every layer: in a log store every layer's block in layer order
-// from offset 0; in a newest-only store each size class's slots for its
-// layers plus its spare (the first pass of layout_slots).
-bool full_step_fits(const lc_store* st, const RangeMap& excl) {
+// Whether the store, empty and with the ranges of `excl` (and of `more`)
+// out of use, takes a step that persists every layer: in a log store every
+// layer's block in layer order from offset 0; in a newest-only store each
+// size class's slots for its layers plus its spare (the first pass of
+// layout_slots).
+bool full_step_fits(const lc_store* st, const RangeMap& excl, const RangeMap& more = RangeMap()) {
     uint64_t top = 0;
     auto put = [&](uint64_t z) {
-        const uint64_t at = place_around(excl, top, z);
+        const uint64_t at = place_around(excl, more, top, z);
         if (at + z > st->capacity) return false;
         top = at + z;
         return true;
@@ -2204,14 +2223,15 @@ extern "C" lc_status lc_store_check_dma(lc_store* st, lc_ctx* ctx, uint64_t regi
     std::stable_sort(slow.begin(), slow.end(),
                      [&](int64_t a, int64_t b) { return worst[size_t(a)] < worst[size_t(b)]; });
     const bool guard = full_step_fits(st, st->excluded);
-    RangeMap trial = st->excluded;
+    RangeMap taken;                      // regions of this call, disjoint from each other
     std::vector<char> take(size_t(n), 0);
     for (int64_t i : slow) {
         const uint64_t off = uint64_t(i) * region_bytes;
-        RangeMap next = trial;
-        add_range(next, off, off + std::min(region_bytes, st->capacity - off));
-        if (guard && !full_step_fits(st, next)) continue;
-        trial.swap(next);
+        taken.emplace(off, std::min(region_bytes, st->capacity - off));
+        if (guard && !full_step_fits(st, st->excluded, taken)) {
+            taken.erase(off);
+            continue;
+        }
         take[size_t(i)] = 1;
     }
     // the slow regions left in use are avoided while a step fits without them
