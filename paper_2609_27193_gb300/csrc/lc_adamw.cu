@@ -224,8 +224,9 @@ __global__ void __launch_bounds__(kMeasureThreads, LC_ADAM_MIN_BLOCKS) adamw_mea
 // model copy with ordinary 16- and 8-byte stores, and add the Eq. 1 sums of
 // the update.  Edge vectors, segments whose arrays do not line up and
 // gradient vectors that would start a bulk copy off a 16-byte boundary go
-// element by element.  Partition, jobs, per-warp partial slots and bounded
-// waits are those of the bulk-load measure.
+// element by element.  Partition (with its pool of units), jobs, the run
+// box that combines the warps' partial sums, and bounded waits are those of
+// the bulk-load measure.
 // ---------------------------------------------------------------------------
 #ifndef LC_ADAM_BULK_STAGES
 #define LC_ADAM_BULK_STAGES 2
@@ -263,16 +264,12 @@ struct ARing {
     uint64_t computed[kAStages];   // consumers done with the buffer (bulk-store form)
     uint64_t empty[kAStages];
     AJob jobs[kAStages];
+    RunBox<kAStages, kAConsumerWarps> box;
 };
 
 __device__ void adam_produce(const MeasureParams& p, const OptSegDev* opt, uint8_t* ring, ARing& r) {
     const uint32_t ring_s = smem_addr(ring);
     const uint32_t full_s = smem_addr(r.full), empty_s = smem_addr(r.empty);
-    const int b = blockIdx.x;
-    int64_t v0 = p.cta_vec_begin[b];
-    const int64_t v1 = p.cta_vec_begin[b + 1];
-    int s = p.cta_seg0[b];
-    int slot = p.cta_slot0[b];
     uint64_t k = 0;
     bool stall = p.stall_first != 0;
     auto post = [&](const AJob& j, const SegDev& sd, const OptSegDev& od) -> bool {
@@ -304,47 +301,54 @@ __device__ void adam_produce(const MeasureParams& p, const OptSegDev* opt, uint8
     bool ok = true;
     SegDev sd{};
     OptSegDev od{};
-    while (ok && v0 < v1 && s < p.nseg) {
-        sd = p.segs[s];
-        od = opt[s];
-        const int64_t seg_end = sd.vec_begin + sd.nvec;
-        const int64_t lo = v0 - sd.vec_begin;
-        const int64_t hi = (v1 < seg_end ? v1 : seg_end) - sd.vec_begin;
-        const bool head_partial = sd.lead > 0;
-        const bool tail_partial = ((int64_t(sd.lead) + sd.numel) % 4) != 0;
-        if (od.fast) {
-            if (head_partial && lo <= 0 && 0 < hi) ok = post({0, 1, kAJobScalar, s, slot, 0}, sd, od);
-            const int64_t kf0 = head_partial ? 1 : 0;
-            const int64_t kf1 = tail_partial ? sd.nvec - 1 : sd.nvec;
-            int64_t x = lo > kf0 ? lo : kf0;
-            const int64_t e = hi < kf1 ? hi : kf1;
-            // a bf16 gradient vector is 8 bytes: a bulk copy must start on 16
-            const uintptr_t gb = uintptr_t(od.grad) - 2 * uintptr_t(sd.lead);
-            if (ok && od.grad_bf16 && x < e && ((gb + 8 * uintptr_t(x)) & 15)) {
-                ok = post({x, x + 1, kAJobScalar, s, slot, 0}, sd, od);
-                ++x;
-            }
-            while (ok && x < e) {
-                int64_t n = e - x < kAChunkVec ? e - x : kAChunkVec;
-                if (od.grad_bf16 && (n & 1)) n -= 1;      // the gradient bytes stay a multiple of 16
-                if (n == 0) {
+    // the CTA's own range, then units of the pool until it is empty
+    for (int rng = int(blockIdx.x); ok && rng >= 0; rng = next_pool_range(p)) {
+        int64_t v0 = p.cta_vec_begin[rng];
+        const int64_t v1 = p.cta_vec_begin[rng + 1];
+        int s = p.cta_seg0[rng];
+        int slot = p.cta_slot0[rng];
+        while (ok && v0 < v1 && s < p.nseg) {
+            sd = p.segs[s];
+            od = opt[s];
+            const int64_t seg_end = sd.vec_begin + sd.nvec;
+            const int64_t lo = v0 - sd.vec_begin;
+            const int64_t hi = (v1 < seg_end ? v1 : seg_end) - sd.vec_begin;
+            const bool head_partial = sd.lead > 0;
+            const bool tail_partial = ((int64_t(sd.lead) + sd.numel) % 4) != 0;
+            if (od.fast) {
+                if (head_partial && lo <= 0 && 0 < hi) ok = post({0, 1, kAJobScalar, s, slot, 0}, sd, od);
+                const int64_t kf0 = head_partial ? 1 : 0;
+                const int64_t kf1 = tail_partial ? sd.nvec - 1 : sd.nvec;
+                int64_t x = lo > kf0 ? lo : kf0;
+                const int64_t e = hi < kf1 ? hi : kf1;
+                // a bf16 gradient vector is 8 bytes: a bulk copy must start on 16
+                const uintptr_t gb = uintptr_t(od.grad) - 2 * uintptr_t(sd.lead);
+                if (ok && od.grad_bf16 && x < e && ((gb + 8 * uintptr_t(x)) & 15)) {
                     ok = post({x, x + 1, kAJobScalar, s, slot, 0}, sd, od);
                     ++x;
-                    continue;
                 }
-                ok = post({x, x + n, kAJobChunk, s, slot, 0}, sd, od);
-                x += n;
+                while (ok && x < e) {
+                    int64_t n = e - x < kAChunkVec ? e - x : kAChunkVec;
+                    if (od.grad_bf16 && (n & 1)) n -= 1;      // the gradient bytes stay a multiple of 16
+                    if (n == 0) {
+                        ok = post({x, x + 1, kAJobScalar, s, slot, 0}, sd, od);
+                        ++x;
+                        continue;
+                    }
+                    ok = post({x, x + n, kAJobChunk, s, slot, 0}, sd, od);
+                    x += n;
+                }
+                const int64_t last = sd.nvec - 1;
+                if (ok && tail_partial && last >= lo && last < hi && !(head_partial && last == 0))
+                    ok = post({last, last + 1, kAJobScalar, s, slot, 0}, sd, od);
+            } else {
+                ok = post({lo, hi, kAJobScalar, s, slot, 0}, sd, od);
             }
-            const int64_t last = sd.nvec - 1;
-            if (ok && tail_partial && last >= lo && last < hi && !(head_partial && last == 0))
-                ok = post({last, last + 1, kAJobScalar, s, slot, 0}, sd, od);
-        } else {
-            ok = post({lo, hi, kAJobScalar, s, slot, 0}, sd, od);
+            if (ok) ok = post({0, 0, kAJobFlush, s, slot, 0}, sd, od);
+            slot += kMeasureBulkSlotsPerRun;
+            ++s;
+            v0 = sd.vec_begin + hi;
         }
-        if (ok) ok = post({0, 0, kAJobFlush, s, slot, 0}, sd, od);
-        slot += kMeasureBulkSlotsPerRun;
-        ++s;
-        v0 = sd.vec_begin + hi;
     }
     if (ok) ok = post({0, 0, kAJobEnd, 0, 0, 0}, sd, od);
     if (!ok) {
@@ -447,7 +451,7 @@ __device__ void adam_consume(const MeasureParams& p, const OptSegDev* opt, const
                 dd += __shfl_down_sync(0xffffffffu, dd, off);
                 da += __shfl_down_sync(0xffffffffu, da, off);
             }
-            if (lane == 0) p.partials[j.slot + warp] = make_double2(dd, da);
+            if (lane == 0) run_box_put<kAConsumerWarps>(r.box, st, warp, dd, da, p.partials + j.slot);
             dd = 0.0;
             da = 0.0;
         }
@@ -458,7 +462,7 @@ __device__ void adam_consume(const MeasureParams& p, const OptSegDev* opt, const
 
 // Bulk-store form: once every consumer warp is done with a buffer, write its
 // updated w, m and v back with bulk stores, and hand the buffer to the
-// producer when those stores have read it.  Its partial slot is zero.
+// producer when those stores have read it.
 __device__ void adam_store(const MeasureParams& p, const OptSegDev* opt, const uint8_t* ring, ARing& r) {
     const uint32_t done_s = smem_addr(r.computed), empty_s = smem_addr(r.empty);
     const uint32_t ring_s = smem_addr(ring);
@@ -489,8 +493,6 @@ __device__ void adam_store(const MeasureParams& p, const OptSegDev* opt, const u
                          : "memory");
             asm volatile("cp.async.bulk.commit_group;" ::: "memory");
             asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
-        } else if (j.kind == kAJobFlush) {
-            p.partials[j.slot + kMeasureBulkSlotsPerRun - 1] = make_double2(0.0, 0.0);
         }
         mbar_arrive(empty_s + 8 * st);
     }
@@ -508,6 +510,7 @@ __global__ void __launch_bounds__(kMeasureThreads, 1) adamw_bulk_kernel(const Me
             mbar_init(smem_addr(&r.full[st]), 1);
             mbar_init(smem_addr(&r.computed[st]), kAConsumerWarps);
             mbar_init(smem_addr(&r.empty[st]), kABulkStore ? 1 : kAConsumerWarps);
+            r.box.count[st] = 0u;
         }
         mbar_init_fence();
     }

@@ -37,6 +37,17 @@ using namespace lc;
 #ifndef LC_COPY_BULK_WAVES
 #define LC_COPY_BULK_WAVES 8
 #endif
+// The bulk measure (and the fused step on its partition): a CTA walks an
+// equal share of the first (100 - LC_MEASURE_POOL_PCT)% of the work space,
+// then takes small units of the rest, LC_MEASURE_POOL_UNITS per CTA in all,
+// from a counter.  CTAs that stream faster take more units, so the launch
+// ends when the pool runs dry rather than when its slowest share is done.
+#ifndef LC_MEASURE_POOL_PCT
+#define LC_MEASURE_POOL_PCT 10
+#endif
+#ifndef LC_MEASURE_POOL_UNITS
+#define LC_MEASURE_POOL_UNITS 8
+#endif
 
 // ---------------------------------------------------------------------------
 // errors
@@ -775,25 +786,35 @@ static lc_status register_layout_impl(lc_ctx* ctx, const lc_segment* segs, int32
     // CTA work ranges of the measure work space: G equal shares in granules
     // of LC_MEASURE_ALIGN_VECS, and `per_run` partial slots for every
     // (CTA, segment) run
+    // (with a pool: G static ranges over the first granules, then `units`
+    // ranges over the rest; range r's slots are fixed whichever CTA walks it)
     struct Partition {
         int64_t G = 0;
+        int64_t units = 0;
         std::vector<int64_t> cta_vec;
         std::vector<int32_t> cta_seg0, cta_slot0, seg_slot_begin;
         int32_t nslots = 0;
     };
-    auto partition = [&](int64_t grid, int32_t per_run) {
+    auto partition = [&](int64_t grid, int32_t per_run, int64_t pool_pct = 0, int64_t units_per_cta = 0) {
         Partition pt;
         const int64_t gran = LC_MEASURE_ALIGN_VECS;
         const int64_t ngran = (V + gran - 1) / gran;
         pt.G = std::max<int64_t>(1, std::min<int64_t>(ngran, grid));
         const int64_t G = pt.G;
-        pt.cta_vec.resize(G + 1);
-        pt.cta_seg0.resize(G);
-        pt.cta_slot0.resize(G);
+        // granules in the pool, in units of at least kMinUnit granules (32 KB)
+        constexpr int64_t kMinUnit = 64;
+        int64_t pool = pool_pct > 0 ? ngran * pool_pct / 100 : 0;
+        pt.units = pool >= kMinUnit ? std::min<int64_t>(G * units_per_cta, pool / kMinUnit) : 0;
+        if (pt.units == 0) pool = 0;
+        const int64_t U = pt.units, R = G + U, ng_static = ngran - pool;
+        pt.cta_vec.resize(R + 1);
+        pt.cta_seg0.resize(R);
+        pt.cta_slot0.resize(R);
         pt.seg_slot_begin.assign(nseg + 1, -1);
-        for (int64_t b = 0; b <= G; ++b) pt.cta_vec[b] = std::min(V, ngran * b / G * gran);
+        for (int64_t b = 0; b <= G; ++b) pt.cta_vec[b] = std::min(V, ng_static * b / G * gran);
+        for (int64_t u = 1; u <= U; ++u) pt.cta_vec[G + u] = std::min(V, (ng_static + pool * u / U) * gran);
         int32_t slot = 0, s = 0;
-        for (int64_t b = 0; b < G; ++b) {
+        for (int64_t b = 0; b < R; ++b) {
             const int64_t v0 = pt.cta_vec[b], v1 = pt.cta_vec[b + 1];
             while (s < nseg && sd[s].vec_begin + sd[s].nvec <= v0) ++s;
             pt.cta_seg0[b] = s;
@@ -814,8 +835,9 @@ static lc_status register_layout_impl(lc_ctx* ctx, const lc_segment* segs, int32
     const Partition pa = partition(int64_t(ctx->sms) * std::max(1, occ), 1);
     int bocc = 0;
     LC_CUDA(measure_bulk_prepare(&bocc));
-    const Partition pb =
-        partition(int64_t(ctx->sms) * std::max(1, bocc) * LC_MEASURE_BULK_WAVES, kMeasureBulkSlotsPerRun);
+    const Partition pb = partition(int64_t(ctx->sms) * std::max(1, bocc) * LC_MEASURE_BULK_WAVES,
+                                   kMeasureBulkSlotsPerRun, LC_MEASURE_POOL_PCT, LC_MEASURE_POOL_UNITS);
+    const int64_t Rb = pb.G + pb.units;
     const int64_t G = pa.G, Gb = pb.G;
     ctx->measure_grid = int(G);
     ctx->measure_bulk_grid = int(Gb);
@@ -882,9 +904,10 @@ static lc_status register_layout_impl(lc_ctx* ctx, const lc_segment* segs, int32
     const size_t o_segsum = tp.take(sizeof(double) * 2 * nseg);
     const size_t o_sums = tp.take(sizeof(double) * 3 * nlayers);
     const size_t o_ticket = tp.take(sizeof(unsigned int));
-    const size_t o_ctav_b = tp.take(sizeof(int64_t) * (Gb + 1));
-    const size_t o_ctas_b = tp.take(sizeof(int32_t) * Gb);
-    const size_t o_ctal_b = tp.take(sizeof(int32_t) * Gb);
+    const size_t o_ctav_b = tp.take(sizeof(int64_t) * (Rb + 1));
+    const size_t o_ctas_b = tp.take(sizeof(int32_t) * Rb);
+    const size_t o_ctal_b = tp.take(sizeof(int32_t) * Rb);
+    const size_t o_unit_b = tp.take(sizeof(unsigned int));
     const size_t o_segslot_b = tp.take(sizeof(int32_t) * (nseg + 1));
     const size_t o_part_b = tp.take(sizeof(double2) * std::max(1, pb.nslots));
     const size_t o_ticket_b = tp.take(sizeof(unsigned int));
@@ -919,9 +942,9 @@ static lc_status register_layout_impl(lc_ctx* ctx, const lc_segment* segs, int32
     put(o_ctas, pa.cta_seg0.data(), sizeof(int32_t) * G);
     put(o_ctal, pa.cta_slot0.data(), sizeof(int32_t) * G);
     put(o_segslot, pa.seg_slot_begin.data(), sizeof(int32_t) * (nseg + 1));
-    put(o_ctav_b, pb.cta_vec.data(), sizeof(int64_t) * (Gb + 1));
-    put(o_ctas_b, pb.cta_seg0.data(), sizeof(int32_t) * Gb);
-    put(o_ctal_b, pb.cta_slot0.data(), sizeof(int32_t) * Gb);
+    put(o_ctav_b, pb.cta_vec.data(), sizeof(int64_t) * (Rb + 1));
+    put(o_ctas_b, pb.cta_seg0.data(), sizeof(int32_t) * Rb);
+    put(o_ctal_b, pb.cta_slot0.data(), sizeof(int32_t) * Rb);
     put(o_segslot_b, pb.seg_slot_begin.data(), sizeof(int32_t) * (nseg + 1));
     put(o_lsb, ctx->layer_seg_begin.data(), sizeof(int32_t) * (nlayers + 1));
     put(o_mult, mult.data(), sizeof(double) * nlayers);
@@ -962,6 +985,8 @@ static lc_status register_layout_impl(lc_ctx* ctx, const lc_segment* segs, int32
     mpb.seg_slot_begin = reinterpret_cast<const int32_t*>(base + o_segslot_b);
     mpb.partials = reinterpret_cast<double2*>(base + o_part_b);
     mpb.ticket = reinterpret_cast<unsigned int*>(base + o_ticket_b);
+    mpb.units = int32_t(pb.units);
+    mpb.unit_next = reinterpret_cast<unsigned int*>(base + o_unit_b);
     mpb.stall_first = (ctx->cfg.debug_flags & LC_DEBUG_MEASURE_STALL) ? 1 : 0;
     ctx->bulk_measure = ctx->cfg.copy_engine == LC_COPY_BULK && all_device && !ctx->snap_missing;
 

@@ -56,6 +56,11 @@ struct MeasureParams {
     // bytes more than it brings)
     uint32_t* fault;
     int32_t stall_first;
+    // bulk kernels: after its own range b (of gridDim.x), a CTA takes the
+    // ranges gridDim.x + u of a pool of `units` small ones, u from
+    // atomicAdd(unit_next, 1), until the pool is empty; 0: no pool
+    int32_t units;
+    unsigned int* unit_next;         // reset by the last CTA
 };
 
 // One copy entry.  The entries of a launch tile a linear "work space"
@@ -199,9 +204,10 @@ cudaError_t launch_measure(const MeasureParams& p, int grid, bool write_ref, cud
 cudaError_t measure_occupancy(int* blocks_per_sm);
 // Bulk-load measure: W and R stream through a shared-memory ring
 // (cp.async.bulk); its partition gives every (CTA, segment) run
-// kMeasureBulkSlotsPerRun consecutive partial slots.  W and R must be
-// device memory.  write_ref: accumulate mode (R <- W as well).
-constexpr int kMeasureBulkSlotsPerRun = kMeasureThreads / 32 - 1;
+// kMeasureBulkSlotsPerRun partial slots (the CTA's consumer warps combine
+// their shares into one).  W and R must be device memory.  write_ref:
+// accumulate mode (R <- W as well).
+constexpr int kMeasureBulkSlotsPerRun = 1;
 cudaError_t launch_measure_bulk(const MeasureParams& p, int grid, bool write_ref, cudaStream_t s);
 cudaError_t measure_bulk_prepare(int* blocks_per_sm);
 cudaError_t launch_adamw_measure(const MeasureParams& p, const OptSegDev* opt, const AdamConsts& c,

@@ -4,12 +4,14 @@
 // Work decomposition: every segment is covered by 16-byte "virtual vectors"
 // aligned to absolute addresses (lc_internal.cuh).  All vectors of all
 // segments, layers ascending, form one linear work space that is cut into
-// G equal contiguous ranges, one per CTA, with G = resident CTAs on the
-// device (one wave).  A CTA streams its range with 128-bit non-allocating
-// loads of W and R, several in flight per thread, and writes one fp64
-// partial per (CTA, segment) run.  The last CTA to finish (atomic ticket, no
-// spinning) adds the partials of each segment, then the segments of each
-// layer, in a fixed order, so the result is deterministic for a layout.
+// contiguous ranges: G equal ones, one per CTA, with G = resident CTAs on
+// the device (one wave), and for the bulk kernel a pool of small ones after
+// them.  A CTA streams its range(s) (the thread kernel: 128-bit
+// non-allocating loads of W and R, several in flight per thread) and writes
+// one fp64 partial per (range, segment) run.  The last CTA to finish (atomic
+// ticket, no spinning) adds the partials of each segment, then the segments
+// of each layer, in a fixed order, so the result is deterministic for a
+// layout.
 //
 // Precision: per-thread fp32 accumulators take at most kUnroll * kFlush
 // terms each before they are added (fixed tree) into per-thread fp64 sums;
@@ -193,9 +195,12 @@ __global__ void __launch_bounds__(kMeasureThreads) measure_kernel(const MeasureP
 }
 
 // ---------------------------------------------------------------------------
-// Bulk-load measure.  The CTA's work range is the same walk over segment
-// runs as above, turned into a sequence of jobs by one producer thread
-// (warp 0): for the full co-aligned vectors of a run, chunks of up to
+// Bulk-load measure.  The CTA walks its own range of the work space and
+// then units of a pool of small ranges, each taken from a counter
+// (next_pool_range), so that CTAs streaming faster take more of the work.
+// Each range is the same walk over segment runs as above, turned into a
+// sequence of jobs by one producer thread (warp 0): for the full co-aligned
+// vectors of a run, chunks of up to
 // kMChunk bytes of W and the same bytes of R loaded by cp.async.bulk into a
 // ring of kMStages buffers (one "full" mbarrier per buffer, completed by the
 // loads' byte count); for partial edge vectors and runs whose W and R are
@@ -203,9 +208,11 @@ __global__ void __launch_bounds__(kMeasureThreads) measure_kernel(const MeasureP
 // element; after each run a flush.  Warps 1..7 consume every job in order:
 // each thread adds its 16-byte vectors of the chunk into fp32 lanes (at most
 // ceil(chunk vectors / 224) terms before they go to fp64), and at a flush
-// each warp reduces its threads' fp64 sums in a fixed order and writes them
-// to its own partial slot of the run, so no barrier spans warps.  Each warp
-// hands a buffer back on its "empty" mbarrier (7 arrivals).  Every wait is
+// each warp reduces its threads' fp64 sums in a fixed order into the run
+// box; the last warp to arrive adds the warps' sums in warp order and
+// writes the run's partial slot (run_box_put), so no warp waits for another
+// and no barrier spans warps.  Each warp hands a buffer back on its "empty"
+// mbarrier (7 arrivals).  Every wait is
 // bounded; a wait that runs out raises the fault word.  Warp-wide decisions
 // (the wait's outcome) are taken by lane 0 and broadcast, so the lanes of a
 // warp never part ways.
@@ -218,7 +225,7 @@ __global__ void __launch_bounds__(kMeasureThreads) measure_kernel(const MeasureP
 #endif
 constexpr int kMStages = LC_MEASURE_BULK_STAGES;
 constexpr uint32_t kMChunk = LC_MEASURE_BULK_CHUNK;      // bytes of W (and of R) per buffer
-constexpr int kMConsumerWarps = kMeasureBulkSlotsPerRun;
+constexpr int kMConsumerWarps = kMeasureThreads / 32 - 1;   // warps 1.. consume (2.. in accumulate mode)
 constexpr int kMConsumers = 32 * kMConsumerWarps;
 constexpr size_t kMeasureBulkSmem = size_t(kMStages) * 2 * kMChunk;
 static_assert(kMChunk % 16 == 0 && kMStages >= 2, "measure ring shape");
@@ -237,16 +244,12 @@ struct MRing {
     uint64_t full[kMStages];
     uint64_t empty[kMStages];
     MJob jobs[kMStages];
+    RunBox<kMStages, kMConsumerWarps> box;
 };
 
 __device__ void measure_produce(const MeasureParams& p, uint8_t* ring, MRing& r) {
     const uint32_t ring_s = smem_addr(ring);
     const uint32_t full_s = smem_addr(r.full), empty_s = smem_addr(r.empty);
-    const int b = blockIdx.x;
-    int64_t v0 = p.cta_vec_begin[b];
-    const int64_t v1 = p.cta_vec_begin[b + 1];
-    int s = p.cta_seg0[b];
-    int slot = p.cta_slot0[b];
     uint64_t k = 0;
     bool stall = p.stall_first != 0;
     auto post = [&](const MJob& j, const SegDev& sd) -> bool {
@@ -271,33 +274,40 @@ __device__ void measure_produce(const MeasureParams& p, uint8_t* ring, MRing& r)
     };
     bool ok = true;
     SegDev sd{};
-    while (ok && v0 < v1 && s < p.nseg) {
-        sd = p.segs[s];
-        const int64_t seg_end = sd.vec_begin + sd.nvec;
-        const int64_t lo = v0 - sd.vec_begin;
-        const int64_t hi = (v1 < seg_end ? v1 : seg_end) - sd.vec_begin;
-        const int ve = 16 >> sd.esz_log2;
-        const bool head_partial = sd.lead > 0;
-        const bool tail_partial = ((int64_t(sd.lead) + sd.numel) % ve) != 0;
-        if (sd.coaligned) {
-            if (head_partial && lo <= 0 && 0 < hi) ok = post({0, 1, kJobScalar, s, slot, 0}, sd);
-            const int64_t kf0 = head_partial ? 1 : 0;
-            const int64_t kf1 = tail_partial ? sd.nvec - 1 : sd.nvec;
-            const int64_t a = lo > kf0 ? lo : kf0;
-            const int64_t e = hi < kf1 ? hi : kf1;
-            constexpr int64_t kCV = kMChunk / 16;
-            for (int64_t x = a; ok && x < e; x += kCV)
-                ok = post({x, (x + kCV < e ? x + kCV : e), kJobChunk, s, slot, sd.esz_log2}, sd);
-            const int64_t last = sd.nvec - 1;
-            if (ok && tail_partial && last >= lo && last < hi && !(head_partial && last == 0))
-                ok = post({last, last + 1, kJobScalar, s, slot, 0}, sd);
-        } else {
-            ok = post({lo, hi, kJobScalar, s, slot, 0}, sd);
+    // the CTA's own range, then units of the pool until it is empty
+    for (int rng = int(blockIdx.x); ok && rng >= 0; rng = next_pool_range(p)) {
+        int64_t v0 = p.cta_vec_begin[rng];
+        const int64_t v1 = p.cta_vec_begin[rng + 1];
+        int s = p.cta_seg0[rng];
+        int slot = p.cta_slot0[rng];
+        while (ok && v0 < v1 && s < p.nseg) {
+            sd = p.segs[s];
+            const int64_t seg_end = sd.vec_begin + sd.nvec;
+            const int64_t lo = v0 - sd.vec_begin;
+            const int64_t hi = (v1 < seg_end ? v1 : seg_end) - sd.vec_begin;
+            const int ve = 16 >> sd.esz_log2;
+            const bool head_partial = sd.lead > 0;
+            const bool tail_partial = ((int64_t(sd.lead) + sd.numel) % ve) != 0;
+            if (sd.coaligned) {
+                if (head_partial && lo <= 0 && 0 < hi) ok = post({0, 1, kJobScalar, s, slot, 0}, sd);
+                const int64_t kf0 = head_partial ? 1 : 0;
+                const int64_t kf1 = tail_partial ? sd.nvec - 1 : sd.nvec;
+                const int64_t a = lo > kf0 ? lo : kf0;
+                const int64_t e = hi < kf1 ? hi : kf1;
+                constexpr int64_t kCV = kMChunk / 16;
+                for (int64_t x = a; ok && x < e; x += kCV)
+                    ok = post({x, (x + kCV < e ? x + kCV : e), kJobChunk, s, slot, sd.esz_log2}, sd);
+                const int64_t last = sd.nvec - 1;
+                if (ok && tail_partial && last >= lo && last < hi && !(head_partial && last == 0))
+                    ok = post({last, last + 1, kJobScalar, s, slot, 0}, sd);
+            } else {
+                ok = post({lo, hi, kJobScalar, s, slot, 0}, sd);
+            }
+            if (ok) ok = post({0, 0, kJobFlush, s, slot, 0}, sd);
+            slot += kMeasureBulkSlotsPerRun;
+            ++s;
+            v0 = sd.vec_begin + hi;
         }
-        if (ok) ok = post({0, 0, kJobFlush, s, slot, 0}, sd);
-        slot += kMeasureBulkSlotsPerRun;
-        ++s;
-        v0 = sd.vec_begin + hi;
     }
     if (ok) ok = post({0, 0, kJobEnd, 0, 0, 0}, sd);
     if (!ok) {
@@ -356,7 +366,8 @@ __device__ void measure_consume(const MeasureParams& p, const uint8_t* ring, MRi
                 dd += __shfl_down_sync(0xffffffffu, dd, off);
                 da += __shfl_down_sync(0xffffffffu, da, off);
             }
-            if (lane == 0) p.partials[j.slot + warp] = make_double2(dd, da);
+            if (lane == 0)
+                run_box_put<kMConsumerWarps - (WRITE_R ? 1 : 0)>(r.box, st, warp, dd, da, p.partials + j.slot);
             dd = 0.0;
             da = 0.0;
         }
@@ -368,7 +379,7 @@ __device__ void measure_consume(const MeasureParams& p, const uint8_t* ring, MRi
 // Accumulate mode (R <- W after the measure, Eq. 1 against W(t-1)): one
 // thread stores every staged W chunk to R with a bulk store once the chunk
 // (and with it the old R) has landed, and hands the buffer back when the
-// store has read it.  Its partial slot of each run is written as zero.
+// store has read it.
 __device__ void measure_store_r(const MeasureParams& p, const uint8_t* ring, MRing& r) {
     const uint32_t full_s = smem_addr(r.full), empty_s = smem_addr(r.empty);
     const uint32_t ring_s = smem_addr(ring);
@@ -389,8 +400,6 @@ __device__ void measure_store_r(const MeasureParams& p, const uint8_t* ring, MRi
                          : "memory");
             asm volatile("cp.async.bulk.commit_group;" ::: "memory");
             asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
-        } else if (j.kind == kJobFlush) {
-            p.partials[j.slot + kMConsumerWarps - 1] = make_double2(0.0, 0.0);
         }
         mbar_arrive(empty_s + 8 * st);
     }
@@ -406,6 +415,7 @@ __global__ void __launch_bounds__(kMeasureThreads, 1) measure_bulk_kernel(const 
         for (int st = 0; st < kMStages; ++st) {
             mbar_init(smem_addr(&r.full[st]), 1);
             mbar_init(smem_addr(&r.empty[st]), kMConsumerWarps);
+            r.box.count[st] = 0u;
         }
         mbar_init_fence();
     }

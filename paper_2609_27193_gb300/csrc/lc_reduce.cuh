@@ -68,6 +68,50 @@ __device__ __forceinline__ void block_sum(double& d, double& a, double* sd, doub
     __syncthreads();
 }
 
+// A run's partial from a bulk kernel's consumer warps.  Each warp's lane 0
+// leaves its warp-reduced (d, a) in the box of the flush job's ring stage;
+// the last of the N contributing warps to arrive adds them in warp order and
+// writes the run's one partial slot.  No warp waits for another.  A stage's
+// box is used again only once every warp has handed that stage back, so
+// warps up to a ring's depth apart never share a box.
+template <int NSTAGES, int MAXW>
+struct RunBox {
+    double d[NSTAGES][MAXW];
+    double a[NSTAGES][MAXW];
+    unsigned int count[NSTAGES];
+};
+
+template <int N, int NSTAGES, int MAXW>
+__device__ __forceinline__ void run_box_put(RunBox<NSTAGES, MAXW>& b, int st, int w, double d, double a,
+                                            double2* slot) {
+    static_assert(N <= MAXW, "run box too small");
+    volatile double* vd = b.d[st];
+    volatile double* va = b.a[st];
+    vd[w] = d;
+    va[w] = a;
+    __threadfence_block();
+    if (atomicAdd(&b.count[st], 1u) == unsigned(N - 1)) {
+        __threadfence_block();
+        double sd = 0.0, sa = 0.0;
+        for (int i = 0; i < N; ++i) {
+            sd += vd[i];
+            sa += va[i];
+        }
+        *slot = make_double2(sd, sa);
+        *reinterpret_cast<volatile unsigned int*>(&b.count[st]) = 0u;
+    }
+}
+
+// The next pool range for the calling CTA (its producer thread), or -1 once
+// the pool is empty.  Asked for only when the CTA's current range has been
+// handed to its consumers, so a unit is claimed by whichever CTA is ready
+// first.
+__device__ __forceinline__ int next_pool_range(const MeasureParams& p) {
+    if (p.units <= 0) return -1;
+    const unsigned int u = atomicAdd(p.unit_next, 1u);
+    return u < unsigned(p.units) ? int(gridDim.x) + int(u) : -1;
+}
+
 // Run by the last CTA: the partial slots of every segment are added, then
 // one thread per layer adds its segments in order.  The order of every
 // addition is fixed by the layout.  The combine runs while the rest of the
@@ -226,7 +270,10 @@ __device__ void finalize(const MeasureParams& p, double2* stage = nullptr, int32
         p.sums[3 * l + 1] = a;
         p.sums[3 * l + 2] = double(n);
     }
-    if (threadIdx.x == 0) *p.ticket = 0u;
+    if (threadIdx.x == 0) {
+        *p.ticket = 0u;
+        if (p.unit_next) *p.unit_next = 0u;   // every CTA has left the pool
+    }
 }
 
 }  // namespace
