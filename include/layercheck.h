@@ -172,6 +172,9 @@ typedef struct {
     uint64_t h2d_bytes;          /* bytes copied host -> device by the library  */
     int64_t bulk_copy_launches;  /* copy launches that ran on the bulk engine   */
     int64_t bulk_measure_launches; /* measure launches on the bulk engine       */
+    int64_t measure_pool_units;    /* small ranges that the bulk measure's CTAs
+                                      take from a pool after their own (0: the
+                                      layout is too small for one)             */
 } lc_counters;
 
 /* Fills cfg with the defaults listed in lc_config. */

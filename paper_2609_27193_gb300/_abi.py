@@ -67,7 +67,8 @@ class lc_counters(C.Structure):
     _fields_ = [("kernel_launches", C.c_int64), ("measure_launches", C.c_int64),
                 ("select_launches", C.c_int64), ("copy_launches", C.c_int64),
                 ("d2h_bytes", C.c_uint64), ("h2d_bytes", C.c_uint64),
-                ("bulk_copy_launches", C.c_int64), ("bulk_measure_launches", C.c_int64)]
+                ("bulk_copy_launches", C.c_int64), ("bulk_measure_launches", C.c_int64),
+                ("measure_pool_units", C.c_int64)]
 
 
 class lc_manifest_record(C.Structure):

@@ -801,10 +801,12 @@ static lc_status register_layout_impl(lc_ctx* ctx, const lc_segment* segs, int32
         const int64_t ngran = (V + gran - 1) / gran;
         pt.G = std::max<int64_t>(1, std::min<int64_t>(ngran, grid));
         const int64_t G = pt.G;
-        // granules in the pool, in units of at least kMinUnit granules (32 KB)
-        constexpr int64_t kMinUnit = 64;
+        // granules in the pool, in units of at least kMinUnit granules (512 KB
+        // of W: a unit costs a counter fetch, a table lookup and a flush); a
+        // pool too small to give every CTA a unit on average is not used
+        constexpr int64_t kMinUnit = 1024;
         int64_t pool = pool_pct > 0 ? ngran * pool_pct / 100 : 0;
-        pt.units = pool >= kMinUnit ? std::min<int64_t>(G * units_per_cta, pool / kMinUnit) : 0;
+        pt.units = pool >= G * kMinUnit ? std::min<int64_t>(G * units_per_cta, pool / kMinUnit) : 0;
         if (pt.units == 0) pool = 0;
         const int64_t U = pt.units, R = G + U, ng_static = ngran - pool;
         pt.cta_vec.resize(R + 1);
@@ -986,6 +988,7 @@ static lc_status register_layout_impl(lc_ctx* ctx, const lc_segment* segs, int32
     mpb.partials = reinterpret_cast<double2*>(base + o_part_b);
     mpb.ticket = reinterpret_cast<unsigned int*>(base + o_ticket_b);
     mpb.units = int32_t(pb.units);
+    ctx->counters.measure_pool_units = pb.units;
     mpb.unit_next = reinterpret_cast<unsigned int*>(base + o_unit_b);
     mpb.stall_first = (ctx->cfg.debug_flags & LC_DEBUG_MEASURE_STALL) ? 1 : 0;
     ctx->bulk_measure = ctx->cfg.copy_engine == LC_COPY_BULK && all_device && !ctx->snap_missing;

@@ -10,8 +10,8 @@ from lc_workloads import gen, shapes
 from lc_workloads.shapes import ModelShape, TensorSpec
 from oracle import oracle as O
 from tests.conftest import GOLDEN
-from tests.lc_harness import (U_RTOL, compare_decision, make_lc, make_oracle, rel_err,
-                              require_gpu)
+from tests.lc_harness import (U_RTOL, compare_decision, make_lc, make_oracle, oracle_measure_parallel,
+                              rel_err, require_gpu)
 
 pytestmark = pytest.mark.gpu
 
@@ -88,6 +88,35 @@ def test_measure_edge_shapes(alloc, dtype, engine):
     lc.measure(1)
     mask, u, _ = lc.select(1e-3, 100)
     ou, _ = run.measure(st.host_all("W"))
+    run.select(ou, 1e-3, 100, 1)
+    compare_decision(mask, u, run, ou, 1e-3)
+    lc.close()
+
+
+@pytest.mark.parametrize("alloc", ["flat", "skew"])
+def test_measure_pool_of_ranges_with_odd_segments(alloc):
+    """The bulk measure's CTAs take small ranges from a pool once their own
+    range is done; unit boundaries then fall anywhere in the work space.
+    About 1.2 G elements in odd-sized segments of mixed dtypes over five
+    layers, packed back to back (flat: most segments start off a 16-byte
+    boundary, W and R alike) or with R shifted by one element (skew: W and R
+    never co-aligned, so every run goes element by element): enough for the
+    library to use a pool, and the sums must match the oracle's."""
+    require_gpu()
+    rng = np.random.default_rng(17)
+    big = [int(x) | 1 for x in rng.integers(20_000_000, 140_000_000, size=14)]
+    small = [1, 3, 7, 33, 4097, 65535, 1000003]
+    sizes = [(n, i % 5) for i, n in enumerate(big[:7] + small + big[7:])]
+    spec = custom_shape(sizes)
+    dts = ["f32" if i % 4 == 1 else "bf16" for i in range(len(sizes))]
+    st = gen.SyntheticState(spec, device="cuda", seed=23, alloc=alloc, dtypes=dts, master=False)
+    st.drift(1, np.array([2e-2, 3e-3, 1e-2, 5e-2, 8e-3]))
+    lc = make_lc(st, copy_engine="bulk")
+    assert lc.counters()["measure_pool_units"] > 0, "layout too small for a pool"
+    run = make_oracle(st)
+    lc.measure(1)
+    mask, u, _ = lc.select(1e-3, 100)
+    ou, _ = oracle_measure_parallel(run, st.host_all("W"))
     run.select(ou, 1e-3, 100, 1)
     compare_decision(mask, u, run, ou, 1e-3)
     lc.close()
