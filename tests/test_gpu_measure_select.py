@@ -93,16 +93,21 @@ def test_measure_edge_shapes(alloc, dtype, engine):
     lc.close()
 
 
+@pytest.mark.parametrize("mode", ["snapshot", "accumulate"])
 @pytest.mark.parametrize("alloc", ["flat", "skew"])
-def test_measure_pool_of_ranges_with_odd_segments(alloc):
+def test_measure_pool_of_ranges_with_odd_segments(alloc, mode):
     """The bulk measure's CTAs take small ranges from a pool once their own
     range is done; unit boundaries then fall anywhere in the work space.
     About 1.2 G elements in odd-sized segments of mixed dtypes over five
     layers, packed back to back (flat: most segments start off a 16-byte
     boundary, W and R alike) or with R shifted by one element (skew: W and R
     never co-aligned, so every run goes element by element): enough for the
-    library to use a pool, and the sums must match the oracle's."""
-    require_gpu()
+    library to use a pool, and the sums must match the oracle's.  In
+    accumulate mode (six consumer warps and a storer that writes R <- W) R
+    must equal W afterwards, bit for bit, in every tensor."""
+    torch = require_gpu()
+    import paper_2609_27193_gb300 as P
+    acc = mode == "accumulate"
     rng = np.random.default_rng(17)
     big = [int(x) | 1 for x in rng.integers(20_000_000, 140_000_000, size=14)]
     small = [1, 3, 7, 33, 4097, 65535, 1000003]
@@ -111,14 +116,19 @@ def test_measure_pool_of_ranges_with_odd_segments(alloc):
     dts = ["f32" if i % 4 == 1 else "bf16" for i in range(len(sizes))]
     st = gen.SyntheticState(spec, device="cuda", seed=23, alloc=alloc, dtypes=dts, master=False)
     st.drift(1, np.array([2e-2, 3e-3, 1e-2, 5e-2, 8e-3]))
-    lc = make_lc(st, copy_engine="bulk")
+    lc = make_lc(st, copy_engine="bulk", mode=P.LC_DRIFT_ACCUMULATE if acc else P.LC_DRIFT_SNAPSHOT)
     assert lc.counters()["measure_pool_units"] > 0, "layout too small for a pool"
-    run = make_oracle(st)
+    run = make_oracle(st, mode=O.ACCUMULATE if acc else O.SNAPSHOT)
     lc.measure(1)
     mask, u, _ = lc.select(1e-3, 100)
     ou, _ = oracle_measure_parallel(run, st.host_all("W"))
     run.select(ou, 1e-3, 100, 1)
     compare_decision(mask, u, run, ou, 1e-3)
+    if acc:
+        torch.cuda.synchronize()
+        for k in range(len(spec.tensors)):
+            bits = torch.int16 if st.W[k].element_size() == 2 else torch.int32
+            assert torch.equal(st.R[k].view(bits), st.W[k].view(bits)), "R <- W of tensor %d" % k
     lc.close()
 
 
