@@ -275,7 +275,7 @@ __device__ void measure_produce(const MeasureParams& p, uint8_t* ring, MRing& r)
     bool ok = true;
     SegDev sd{};
     // the CTA's own range, then units of the pool until it is empty
-    for (int rng = int(blockIdx.x); ok && rng >= 0; rng = next_pool_range(p)) {
+    for (int rng = int(blockIdx.x); ok && rng >= 0; rng = ok ? next_pool_range(p) : -1) {
         int64_t v0 = p.cta_vec_begin[rng];
         const int64_t v1 = p.cta_vec_begin[rng + 1];
         int s = p.cta_seg0[rng];
