@@ -671,11 +671,11 @@ def run_ours(args):
     import numpy as np
     import torch
     rank, world, local = dist_env()
+    torch.cuda.set_device(local)          # before the process group, so NCCL binds this rank's GPU
+    dev = torch.device("cuda", local)
     if world > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl")
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
     P = load_package()
     from lc_workloads import gen
     from lc_workloads import shapes
