@@ -1014,44 +1014,48 @@ def run_ours(args):
         link_streams = d2h_streams_probe(torch, dev)
         e_s = sum(r["host_s"] for r in e_recs)
         e_tot = float(sum(e_bytes))
-        if not e_recs:
-            raise SystemExit("bench: every timed e2e step persisted more than the %.1f GB host store holds "
-                             "(--host-store-gb)" % (cap / 1e9))
-        d2h = statistics.mean(r["nbytes"] for r in e_recs)
         e_tot, e_s = whole_job(e_tot, e_s, world, dev)
-        e2e = {"value": e_tot / e_s / 1e9, "unit": "GB/s", "h2d_bytes_per_step": 0,
-               "d2h_bytes_per_step": int(d2h),
-               "ms_per_step": 1e3 * e_s / len(e_recs),
-               # steps whose layers did not fit a store smaller than a full step
-               # (--host-store-gb, or a host without room for one per rank)
-               "steps_spilled_to_device": spilled,
-               "d2h_GBps": d2h / (statistics.mean((r["host_s"] - r["decision_s"]) if not graph
-                                                  else r["host_s"] for r in e_recs)) / 1e9,
-               # the host link and host memory are shared with other jobs on the
-               # machine: the same copy has measured 50-193 GB/s minutes apart, so
-               # the link is probed right before and right after the loop
-               "d2h_link_GBps_measured": link,
-               "store_dma_check": dma_check,
-               "d2h_link_GBps_after": link_after,
-               # GB/s by number of concurrent copy streams: the link, not the
-               # number of copy engines in use, sets the rate
-               "d2h_link_GBps_by_streams": link_streams,
-               "steps_d2h_ms": [round(1e3 * ((r["host_s"] - r["decision_s"]) if not graph else r["host_s"]), 3)
-                                for r in e_recs],
-               "steps_d2h_bytes": [int(r["nbytes"]) for r in e_recs],
-               # the library's own per-chunk events: D2H spans on its copy
-               # stream (busy = copying, idle = waiting for a gathered chunk)
-               # and the gathers into the staging slots on the context stream
-               "d2h_trace": merge_span_summaries([r.get("d2h_trace") for r in e_recs]),
-               "gather_trace": merge_span_summaries([r.get("gather_trace") for r in e_recs]),
-               "steps_d2h_busy_GBps": [round(r["d2h_trace"]["busy_GBps"], 1) if r.get("d2h_trace") else None
-                                       for r in e_recs],
-               "steps_d2h_idle_ms": [round(r["d2h_trace"]["idle_ms"], 2) if r.get("d2h_trace") else None
-                                     for r in e_recs],
-               "note": "weights, snapshot and moments are device-resident training state; the "
-                       "step's only host traffic is the decision block and the persisted "
-                       "layers copied into %s" % ("pinned host memory by the replayed graph's pack"
-                                                  if graph else "the pinned store")}
+        if not e_recs or e_s <= 0.0:
+            # every timed step persisted more than the host store holds
+            e2e = {"skipped": "every timed step persisted more than the %.1f GB pinned store holds "
+                              "(host memory or --host-store-gb)" % (cap / 1e9),
+                   "steps_spilled_to_device": spilled, "store_dma_check": dma_check}
+            e_recs = None
+        d2h = statistics.mean(r["nbytes"] for r in e_recs) if e_recs else 0
+        if e_recs:
+            e2e = {"value": e_tot / e_s / 1e9, "unit": "GB/s", "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": int(d2h),
+                   "ms_per_step": 1e3 * e_s / len(e_recs),
+                   # steps whose layers did not fit a store smaller than a full step
+                   # (--host-store-gb, or a host without room for one per rank)
+                   "steps_spilled_to_device": spilled,
+                   "d2h_GBps": d2h / (statistics.mean((r["host_s"] - r["decision_s"]) if not graph
+                                                      else r["host_s"] for r in e_recs)) / 1e9,
+                   # the host link and host memory are shared with other jobs on the
+                   # machine: the same copy has measured 50-193 GB/s minutes apart, so
+                   # the link is probed right before and right after the loop
+                   "d2h_link_GBps_measured": link,
+                   "store_dma_check": dma_check,
+                   "d2h_link_GBps_after": link_after,
+                   # GB/s by number of concurrent copy streams: the link, not the
+                   # number of copy engines in use, sets the rate
+                   "d2h_link_GBps_by_streams": link_streams,
+                   "steps_d2h_ms": [round(1e3 * ((r["host_s"] - r["decision_s"]) if not graph else r["host_s"]), 3)
+                                    for r in e_recs],
+                   "steps_d2h_bytes": [int(r["nbytes"]) for r in e_recs],
+                   # the library's own per-chunk events: D2H spans on its copy
+                   # stream (busy = copying, idle = waiting for a gathered chunk)
+                   # and the gathers into the staging slots on the context stream
+                   "d2h_trace": merge_span_summaries([r.get("d2h_trace") for r in e_recs]),
+                   "gather_trace": merge_span_summaries([r.get("gather_trace") for r in e_recs]),
+                   "steps_d2h_busy_GBps": [round(r["d2h_trace"]["busy_GBps"], 1) if r.get("d2h_trace") else None
+                                           for r in e_recs],
+                   "steps_d2h_idle_ms": [round(r["d2h_trace"]["idle_ms"], 2) if r.get("d2h_trace") else None
+                                         for r in e_recs],
+                   "note": "weights, snapshot and moments are device-resident training state; the "
+                           "step's only host traffic is the decision block and the persisted "
+                           "layers copied into %s" % ("pinned host memory by the replayed graph's pack"
+                                                      if graph else "the pinned store")}
         if store is not None and cap >= full:
             e2e["restore"] = restore_leg(torch, dev, P, lc, store, t + 1, tau, full,
                                          trace_file=args.copy_trace)
