@@ -7,9 +7,10 @@ lc_measure without an lc_ctx; its scratch lives in a fixed-size static
 device array.  These tests call it through the C ABI and compare its sums
 with the oracle's, element by element within the tolerance of the measure
 parity tests, on two calls in a row with different inputs (stale scratch
-from the first call would show), on segments passed in shuffled layer
-order, and at exactly LC_NOALLOC_MAX_SEGMENTS segments.  The file is named
-to be collected last."""
+from the first call would show), with lc_measure's sums on the same tensors
+in those two calls, on segments passed in shuffled layer order, and at
+exactly LC_NOALLOC_MAX_SEGMENTS segments.  The file is named to be collected
+last."""
 import ctypes as C
 
 import numpy as np
@@ -17,7 +18,7 @@ import pytest
 
 from lc_workloads import gen, shapes
 from lc_workloads.shapes import ModelShape, TensorSpec
-from tests.lc_harness import U_RTOL, make_oracle, oracle_measure_parallel, require_gpu
+from tests.lc_harness import U_RTOL, make_lc, make_oracle, oracle_measure_parallel, require_gpu
 
 pytestmark = pytest.mark.gpu
 
@@ -37,15 +38,19 @@ def _call(torch, lib, _abi, stream, segs, nseg, nlayers):
     return out.cpu().numpy().reshape(-1, 3)
 
 
-def _check_against_oracle(got, st, what):
-    run = make_oracle(st)
-    _, want = oracle_measure_parallel(run, st.host_all("W"))
+def _check_sums(got, want, what):
     assert np.all(np.isfinite(got)), "%s: a sum was not written" % what
     assert np.array_equal(got[:, 2], want[:, 2]), "%s: element counts differ" % what
     for col in (0, 1):
         den = np.maximum(np.abs(want[:, col]), 1e-300)
         rel = np.abs(got[:, col] - want[:, col]) / den
         assert rel.max() <= U_RTOL, (what, col, int(rel.argmax()), rel.max())
+
+
+def _check_against_oracle(got, st, what):
+    run = make_oracle(st)
+    _, want = oracle_measure_parallel(run, st.host_all("W"))
+    _check_sums(got, want, what)
 
 
 def test_noalloc_measure_matches_oracle_on_two_calls():
@@ -63,15 +68,25 @@ def test_noalloc_measure_matches_oracle_on_two_calls():
     segs = _segments(P, _abi, st, order)
     stream = torch.cuda.Stream()
     scales = np.geomspace(1e-4, 3e-2, N)
+    # the existing entry point on the same tensors, its sums in a buffer of ours
+    lc = make_lc(st)
+    ref = torch.zeros(3 * N, dtype=torch.float64, device="cuda")
+    lc.set_layer_sums_buffer(ref)
     previous = None
     for t in (1, 2):
         st.drift(t, scales)
         torch.cuda.synchronize()
         got = _call(torch, lib, _abi, stream, segs, n, N)
         _check_against_oracle(got, st, "step %d" % t)
+        lc.measure(t)
+        lc.select(1e300, 1 << 30)          # persists nothing: R stays, the drift grows
+        lc.commit_snapshot()
+        torch.cuda.synchronize()
+        _check_sums(got, ref.cpu().numpy().reshape(-1, 3), "lc_measure at step %d" % t)
         if previous is not None:
             assert not np.array_equal(previous[:, 0], got[:, 0]), "second call returned the first's sums"
         previous = got.copy()
+    lc.close()
 
 
 def test_noalloc_at_the_segment_limit():
